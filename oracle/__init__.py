@@ -1,0 +1,8 @@
+"""fp64 CPU oracle for the Nexus splice / re-rotate / suffix-attention path.
+
+TEST INFRASTRUCTURE. Only ``tests/``, ``__graft_entry__.smoke()`` and the CPU
+baseline / reference arm of ``bench.py`` may import this package. It shares no
+code with the CUDA library, and the product path never calls it.
+"""
+from .nexus_oracle import *  # noqa: F401,F403
+from .nexus_oracle import __all__  # noqa: F401

@@ -1,0 +1,149 @@
+"""Seeded synthetic workloads shaped like Qwen2.5-14B attention.
+
+This module only draws random numbers and fixes shapes. It holds none of the
+splice, rotation, policy or attention arithmetic, and both the CUDA path and
+the fp64 oracle take their inputs from it.
+
+Recipe (all values bf16 from float32 N(0, 1), round-to-nearest-even):
+
+* live K/V of each session: N(0, 1) rows, read as keys already rotated at
+  their positions (a rotation maps N(0, I) to N(0, I));
+* compiled schema blocks: N(0, 1) rows compiled at anchor ``base_pos``;
+* queries: N(0, 1) rows, read as already rotated at their positions;
+* integers (block lengths, depths, context lengths, page order) from a
+  NumPy PCG64 generator seeded per workload.
+
+Named workloads (Hq = 40, Hkv = 8, d = 128, 16-token pages):
+
+* ``c1``  1 layer, n_past 512, one 128-token block (anchor 0) at depth 300,
+  64 suffix queries over the 640-token cache;
+* ``c2``  1 layer, n_past 4096, 16 blocks of U{64..512} tokens appended back to
+  back at the cursor, suffix of 25 % of the spliced span;
+* ``c3``  48 layers, n_past 8192, one 1024-token block at depth 6000,
+  transposed-V cache, suffix of {25, 50, 100} % of the 2192 displaced rows;
+* ``c4``  32 sessions x 48 layers, n_past log-uniform in [1024, 16384], four
+  blocks of U{128..768} tokens at sorted U{0..n_past} depths, suffix 50 % of
+  the spliced span, pool pages handed out in a shuffled order;
+* ``c5``  48 layers, n_past 32768, one 2048-token block at depth 30000; a full
+  causal re-prefill of the 32768-token context and a 64-query suffix over the
+  34816-token spliced cache.
+"""
+from __future__ import annotations
+
+import dataclasses
+import math
+from typing import List, Optional
+
+import numpy as np
+import torch
+
+N_Q_HEADS = 40
+N_KV_HEADS = 8
+HEAD_DIM = 128
+PAGE_SIZE = 16
+ROPE_THETA = 1.0e6
+
+
+@dataclasses.dataclass
+class Insert:
+    depth: int        # position in the pre-splice sequence
+    length: int       # block tokens
+    base_pos: int     # compile anchor m0 of the block's first token
+
+
+@dataclasses.dataclass
+class Session:
+    n_past: int
+    inserts: List[Insert]
+    suffix_span: int          # S, the span the redecode fraction applies to
+    suffix_pct: int           # fixed redecode percentage of S for this workload
+
+
+@dataclasses.dataclass
+class Workload:
+    name: str
+    n_layers: int
+    sessions: List[Session]
+    v_transposed: bool = False
+    shuffle_pages: bool = False
+    seed: int = 0
+    suffix_pcts: tuple = ()           # extra percentages swept (c3)
+    reprefill: bool = False           # c5: causal self-attention of the pre-splice context
+    n_q_heads: int = N_Q_HEADS
+    n_kv_heads: int = N_KV_HEADS
+    head_dim: int = HEAD_DIM
+    page_size: int = PAGE_SIZE
+    rope_theta: float = ROPE_THETA
+
+    @property
+    def group(self) -> int:
+        return self.n_q_heads // self.n_kv_heads
+
+    def spliced_len(self, s: Session) -> int:
+        return s.n_past + sum(i.length for i in s.inserts)
+
+
+def _rng(seed: int) -> np.random.Generator:
+    return np.random.Generator(np.random.PCG64(seed))
+
+
+def workload(name: str, n_layers: Optional[int] = None) -> Workload:
+    """One of the named workloads; ``n_layers`` overrides the layer count (tests)."""
+    name = name.lower()
+    if name == "c1":
+        w = Workload("c1", 1, [Session(512, [Insert(300, 128, 0)], 64, 100)], seed=1)
+    elif name == "c2":
+        r = _rng(2)
+        lens = r.integers(64, 512, size=16, endpoint=True)
+        ins = [Insert(4096, int(L), 0) for L in lens]
+        w = Workload("c2", 1, [Session(4096, ins, int(lens.sum()), 25)], seed=2)
+    elif name == "c3":
+        w = Workload("c3", 48, [Session(8192, [Insert(6000, 1024, 0)], 2192, 25)],
+                     v_transposed=True, seed=3, suffix_pcts=(25, 50, 100))
+    elif name == "c4":
+        r = _rng(4)
+        sessions = []
+        for _ in range(32):
+            n_past = int(math.floor(math.exp(r.uniform(math.log(1024), math.log(16384)))))
+            lens = r.integers(128, 768, size=4, endpoint=True)
+            depths = np.sort(r.integers(0, n_past, size=4, endpoint=True))
+            ins = [Insert(int(p), int(L), 0) for p, L in zip(depths, lens)]
+            sessions.append(Session(n_past, ins, int(lens.sum()), 50))
+        w = Workload("c4", 48, sessions, shuffle_pages=True, seed=4)
+    elif name == "c5":
+        w = Workload("c5", 48, [Session(32768, [Insert(30000, 2048, 0)], 64, 100)],
+                     seed=5, reprefill=True)
+    else:
+        raise KeyError(f"unknown workload {name!r}")
+    if n_layers is not None:
+        w.n_layers = int(n_layers)
+    return w
+
+
+def page_order(n_pages: int, seed: int, shuffle: bool) -> np.ndarray:
+    """Order in which a pool hands out its pages: identity, or a seeded permutation."""
+    if not shuffle:
+        return np.arange(n_pages, dtype=np.int32)
+    return _rng(seed + 1000).permutation(n_pages).astype(np.int32)
+
+
+def randn_bf16(shape, seed: int, device="cpu") -> torch.Tensor:
+    """float32 N(0, 1) from a seeded torch generator, rounded to bf16.
+
+    Large tensors are drawn in slices along dim 0 so the float32 staging stays
+    small; each slice has its own derived seed, so the result depends only on
+    (shape, seed), not on the device memory available.
+    """
+    shape = tuple(int(s) for s in shape)
+    out = torch.empty(shape, dtype=torch.bfloat16, device=device)
+    if out.numel() == 0:
+        return out
+    per = max(1, out[0].numel() if len(shape) > 0 else 1)
+    chunk = max(1, (1 << 26) // per)
+    for i0 in range(0, shape[0], chunk):
+        i1 = min(shape[0], i0 + chunk)
+        g = torch.Generator(device=device)
+        g.manual_seed(int(seed) * 1_000_003 + i0)
+        out[i0:i1] = torch.randn((i1 - i0,) + shape[1:], generator=g, device=device,
+                                 dtype=torch.float32).to(torch.bfloat16)
+    return out

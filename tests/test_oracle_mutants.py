@@ -1,0 +1,176 @@
+"""Planted mistakes in copies of the oracle must each trip at least one pin.
+
+Each mutant below is a plausible slip when writing the oracle from the paper
+(a dropped term, a wrong sign, a wrong index, a transposed operand). The
+mutants live here, on the CPU, and never touch the real oracle module.
+"""
+import math
+from fractions import Fraction
+
+import numpy as np
+import pytest
+
+import oracle
+import oracle_pins as P
+
+
+def _fails(fn, *args):
+    try:
+        fn(*args)
+    except AssertionError:
+        return True
+    except Exception:
+        return True
+    return False
+
+
+# ---- policy mutants (Eq. 2)
+def pct_denominator_mk(n, M=256, R_base=5, K=4):
+    if n <= M:
+        return Fraction(R_base)
+    return min(Fraction(R_base) + Fraction(n - M, M * K) * (100 - R_base), Fraction(100))
+
+
+def pct_no_clamp(n, M=256, R_base=5, K=4):
+    if n <= M:
+        return Fraction(R_base)
+    return Fraction(R_base) + Fraction(n - M, M * (K - 1)) * (100 - R_base)
+
+
+def pct_drops_base(n, M=256, R_base=5, K=4):
+    if n <= M:
+        return Fraction(R_base)
+    return min(Fraction(R_base) + Fraction(n - M, M * (K - 1)) * 100, Fraction(100))
+
+
+def len_floor(S, n, M=256, R_base=5, K=4):
+    return min(S, math.floor(Fraction(S) * oracle.recompute_pct(n, M, R_base, K) / 100))
+
+
+@pytest.mark.parametrize("mut", [pct_denominator_mk, pct_no_clamp, pct_drops_base])
+def test_policy_mutants_caught(mut):
+    assert _fails(P.pin_table1, mut) or _fails(P.pin_eq2_shape, mut)
+
+
+def test_redecode_floor_caught():
+    assert _fails(P.pin_redecode_len, len_floor, oracle.recompute_pct)
+
+
+# ---- RoPE mutants
+def _rope_factory(sign=1.0, pairs="half", exponent=2.0, swap_out=False):
+    def rope(x, pos, theta_base=1.0e6, freq_scale=1.0, rope_type="neox"):
+        x = np.asarray(x, dtype=np.float64)
+        d = x.shape[-1]
+        h = d // 2
+        th = freq_scale * theta_base ** (-exponent * np.arange(h) / d)
+        ang = np.asarray(pos, dtype=np.float64)[..., None] * th
+        c, s = np.cos(ang), sign * np.sin(ang)
+        out = np.empty(np.broadcast_shapes(x.shape, ang.shape[:-1] + (d,)))
+        if rope_type == "neox" and pairs == "half":
+            a, b = x[..., :h], x[..., h:]
+            out[..., :h] = a * c - b * s
+            out[..., h:] = (b * s + a * c) if swap_out else (a * s + b * c)
+        else:
+            a, b = x[..., 0::2], x[..., 1::2]
+            out[..., 0::2] = a * c - b * s
+            out[..., 1::2] = a * s + b * c
+        return out
+    return rope
+
+
+ROPE_MUTANTS = {
+    "sin_sign": _rope_factory(sign=-1.0),
+    "interleaved_as_neox": _rope_factory(pairs="interleaved"),
+    "exponent_i_over_d": _rope_factory(exponent=1.0),
+    "swapped_terms": _rope_factory(swap_out=True),
+}
+
+
+@pytest.mark.parametrize("name", sorted(ROPE_MUTANTS))
+def test_rope_mutants_caught(name):
+    m = ROPE_MUTANTS[name]
+    assert (_fails(P.pin_rope_complex, m) or _fails(P.pin_rope_2x2, m)
+            or _fails(P.pin_rope_group, m))
+
+
+# ---- splice mutants
+def splice_tail_not_rotated(live_k, live_v, inserts, *a, **kw):
+    ks, vs, cur, shift = [], [], 0, 0
+    for p, bk, bv, m0 in inserts:
+        ks.append(live_k[:, cur:p]); vs.append(live_v[:, cur:p])
+        ks.append(oracle.rerotate(bk, p + shift - m0)); vs.append(bv)
+        shift += bk.shape[1]; cur = p
+    ks.append(live_k[:, cur:]); vs.append(live_v[:, cur:])
+    return np.concatenate(ks, 1), np.concatenate(vs, 1)
+
+
+def splice_delta_sign(live_k, live_v, inserts, *a, **kw):
+    ks, vs, cur, shift = [], [], 0, 0
+    for p, bk, bv, m0 in inserts:
+        ks.append(oracle.rerotate(live_k[:, cur:p], shift)); vs.append(live_v[:, cur:p])
+        ks.append(oracle.rerotate(bk, m0 - (p + shift))); vs.append(bv)
+        shift += bk.shape[1]; cur = p
+    ks.append(oracle.rerotate(live_k[:, cur:], shift)); vs.append(live_v[:, cur:])
+    return np.concatenate(ks, 1), np.concatenate(vs, 1)
+
+
+def splice_ignores_earlier_inserts(live_k, live_v, inserts, *a, **kw):
+    ks, vs, cur, shift = [], [], 0, 0
+    for p, bk, bv, m0 in inserts:
+        ks.append(oracle.rerotate(live_k[:, cur:p], shift)); vs.append(live_v[:, cur:p])
+        ks.append(oracle.rerotate(bk, p - m0)); vs.append(bv)
+        shift += bk.shape[1]; cur = p
+    ks.append(oracle.rerotate(live_k[:, cur:], shift)); vs.append(live_v[:, cur:])
+    return np.concatenate(ks, 1), np.concatenate(vs, 1)
+
+
+@pytest.mark.parametrize("mut", [splice_tail_not_rotated, splice_delta_sign, splice_ignores_earlier_inserts])
+def test_splice_mutants_caught(mut):
+    assert _fails(P.pin_splice_closed_form, mut, oracle.rope_rotate)
+
+
+def test_rerotate_arithmetic_at_zero_caught():
+    def rerot_always_math(k, delta, *a, **kw):
+        return oracle.rope_rotate(k, int(delta))
+    assert _fails(P.pin_rerotate, rerot_always_math, oracle.rope_rotate)
+
+
+# ---- attention mutants
+def _attn_factory(scale=True, strict=False, head_map="div", transpose_v=False):
+    def attn(q, k, v, q_pos, group):
+        q = np.asarray(q, float); k = np.asarray(k, float); v = np.asarray(v, float)
+        R, Hq, d = q.shape
+        T = k.shape[0]
+        Hkv = k.shape[1]
+        pos = np.asarray(q_pos)
+        vis = (np.arange(T)[None, :] < pos[:, None]) if strict else (np.arange(T)[None, :] <= pos[:, None])
+        o = np.zeros((R, Hq, d)); lse = np.zeros((R, Hq))
+        for h in range(Hq):
+            kv = h // group if head_map == "div" else h % Hkv
+            s = q[:, h] @ k[:, kv].T
+            if scale:
+                s = s / math.sqrt(d)
+            s = np.where(vis, s, -np.inf)
+            m = s.max(1, keepdims=True)
+            e = np.exp(s - m)
+            z = e.sum(1, keepdims=True)
+            vv = v[:, kv]
+            if transpose_v and T == d:
+                vv = vv.T
+            o[:, h] = (e / z) @ vv
+            lse[:, h] = m[:, 0] + np.log(z[:, 0])
+        return o, lse
+    return attn
+
+
+ATTN_MUTANTS = {
+    "no_scale": _attn_factory(scale=False),
+    "strict_mask": _attn_factory(strict=True),
+    "head_mod": _attn_factory(head_map="mod"),
+}
+
+
+@pytest.mark.parametrize("name", sorted(ATTN_MUTANTS))
+def test_attention_mutants_caught(name):
+    m = ATTN_MUTANTS[name]
+    assert (_fails(P.pin_attention_library, m) or _fails(P.pin_attention_special, m))
