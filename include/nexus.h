@@ -1,0 +1,316 @@
+/*
+ * nexus.h - C ABI of the GB300 (sm_103a) KV-cache splicing hot path.
+ *
+ * The operations follow "Nexus: Depth-Adaptive KV-Cache Splicing and
+ * Retrieval-Decoupled Tool Routing for Agentic LLMs on Unified Memory":
+ *
+ *   nexus_splice_kv          write compiled schema K/V rows into a live paged
+ *                            cache at the runtime cursor, reanchoring K by
+ *                            delta = position - base_pos (Sec. III-B, Sec. V-A),
+ *                            row-major or token-innermost V (Sec. V-B)
+ *   nexus_rope_rerotate      rotate cached keys by a position offset
+ *                            (Sec. III-B, Eq. 1)
+ *   nexus_copy_pages         bit-exact page copies (the in-arena KV copy of
+ *                            Sec. V-D)
+ *   nexus_suffix_attention   causal GQA attention of the last R positions over
+ *                            the spliced cache: the redecoded suffix of
+ *                            Sec. III-C / Sec. V-A, softmax(QK^T/sqrt(d))V of
+ *                            Sec. III-A
+ *   nexus_reprefill          the same with R = T: the full re-prefill that
+ *                            R(n_past) = 100 % amounts to (Sec. III-C)
+ *   nexus_recompute_pct, nexus_redecode_len, nexus_check_splice
+ *                            the depth-adaptive policy of Eq. 2 and the
+ *                            splice threshold P (Sec. III-B, Sec. III-C)
+ *   nexus_page_pool_*, nexus_plan_splice
+ *                            host page allocator and splice planner
+ *
+ * Conventions
+ *   - Device buffers are owned by the caller. The library never allocates or
+ *     frees device memory and keeps no per-call state; it caches per-device
+ *     properties and one error word per device.
+ *   - Every call validates its arguments on the host before any launch and
+ *     reports problems as a nexus_status; no exception crosses the ABI.
+ *   - Device calls are asynchronous on the given stream (a cudaStream_t passed
+ *     as void*; NULL is the legacy default stream). A failed launch returns
+ *     NEXUS_ECUDA. nexus_device_status() synchronises a stream and reports
+ *     whether any bounded device wait gave up.
+ *   - Only head_dim = 128, page_size = 16 and bf16 data are accepted.
+ *   - Layouts (all bf16, innermost last):
+ *       K pool        [n_layers][n_pages][n_kv_heads][page_size][head_dim]
+ *       V pool        same, or, when v_transposed,
+ *                     [n_layers][n_pages][n_kv_heads][head_dim][page_size]
+ *       block K / V   [n_layers][n_tokens][n_kv_heads][head_dim]
+ *       page tables   int32 [n_rows][max_pages]; position t of row r lives in
+ *                     page table[r][t / 16], slot t % 16
+ *       Q, O          [n_layers_call][sum of q_len][n_q_heads][head_dim]
+ *       LSE           float [n_layers_call][sum of q_len][n_q_heads]
+ *     Pointers passed for device data must be 16-byte aligned.
+ */
+#ifndef NEXUS_H
+#define NEXUS_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define NEXUS_VERSION 1
+
+typedef void* nexus_stream; /* cudaStream_t */
+
+typedef enum nexus_status {
+  NEXUS_OK = 0,
+  NEXUS_EINVAL = 1,          /* malformed argument (null pointer, bad count, unsupported shape) */
+  NEXUS_ERANGE = 2,          /* a position, page id, row or layer lies outside its table */
+  NEXUS_EROPE_MISMATCH = 3,  /* block RoPE parameters differ from the cache's; the block is
+                                rejected rather than spliced (Sec. V-A) */
+  NEXUS_ELAYOUT = 4,         /* shape or alignment check of a buffer failed (Sec. V-B) */
+  NEXUS_ENOMEM = 5,          /* page pool exhausted, workspace or output capacity too small */
+  NEXUS_EDECLINED = 6,       /* splice past the threshold P without the redecode Eq. 2 asks
+                                for (Sec. III-B) */
+  NEXUS_ECUDA = 7,           /* a CUDA runtime or driver call failed */
+  NEXUS_ETIMEOUT = 8,        /* a bounded device-side wait gave up; results are invalid */
+  NEXUS_EOVERLAP = 9         /* destination rows overlap each other or the source rows */
+} nexus_status;
+
+enum { NEXUS_ROPE_NEOX = 0, NEXUS_ROPE_GPTJ = 1 };
+
+/* Live paged KV cache. RoPE parameters are those of the runtime model; a
+ * block is spliced only if its header carries the same ones (Sec. V-A). */
+typedef struct nexus_kv_cache {
+  void* k_pool;             /* device */
+  void* v_pool;             /* device */
+  int64_t n_pages;          /* pages per layer */
+  int32_t n_layers;
+  int32_t n_kv_heads;
+  int32_t head_dim;         /* 128 */
+  int32_t page_size;        /* 16 */
+  int32_t v_transposed;     /* 0: row-major V; 1: token-innermost V (Sec. V-B) */
+  int32_t rope_type;        /* NEXUS_ROPE_NEOX (half-split pairs) or NEXUS_ROPE_GPTJ */
+  double rope_theta;        /* base b of theta_i = b^(-2i/d); 1e6 (Sec. III-B) */
+  double rope_freq_scale;   /* linear position scale; 1.0 */
+} nexus_kv_cache;
+
+/* Device-resident analogue of a compiled tool block (Sec. V-A): its header
+ * fields and its K/V tensors. Token j of the block was rotated at base_pos + j. */
+typedef struct nexus_block {
+  const void* k;            /* device [n_layers][n_tokens][n_kv_heads][head_dim] */
+  const void* v;            /* device, same shape */
+  int32_t n_tokens;
+  int32_t base_pos;         /* RoPE anchor m0 */
+  int32_t n_layers;
+  int32_t n_kv_heads;
+  int32_t head_dim;
+  int32_t rope_type;
+  double rope_theta;
+  double rope_freq_scale;
+} nexus_block;
+
+enum { NEXUS_SRC_BLOCK = 0, NEXUS_SRC_CACHE = 1 };
+enum { NEXUS_SEG_K_ONLY = 1 };
+
+/* One run of destination rows written by nexus_splice_kv. */
+typedef struct nexus_splice_segment {
+  int32_t src_kind;         /* NEXUS_SRC_BLOCK or NEXUS_SRC_CACHE */
+  int32_t src_index;        /* block index, or page-table row of the source sequence */
+  int32_t src_start;        /* first block token, or first source position */
+  int32_t dst_row;          /* page-table row of the destination sequence */
+  int32_t dst_start;        /* first destination position */
+  int32_t n_tokens;
+  int32_t delta;            /* RoPE offset applied to K; 0 copies the bits (Sec. IV-A) */
+  int32_t flags;            /* NEXUS_SEG_K_ONLY leaves V untouched */
+} nexus_splice_segment;
+
+/* Splice policy: threshold P = M, base fraction R_base and full-recompute
+ * multiple K of Eq. 2 (paper defaults 256, 5, 4; tuned K = 16). */
+typedef struct nexus_policy {
+  int32_t splice_threshold; /* M = P */
+  int32_t r_base_pct;       /* R_base in percent */
+  int32_t full_mult;        /* K >= 2 */
+} nexus_policy;
+
+typedef struct nexus_insert {
+  int32_t depth;            /* position in the pre-splice sequence, non-decreasing */
+  int32_t block_index;      /* index into the blocks array */
+} nexus_insert;
+
+typedef struct nexus_page_pool nexus_page_pool;
+
+/* ---------------------------------------------------------------- status */
+const char* nexus_status_string(nexus_status s);
+int32_t nexus_version(void);
+
+/* Synchronises `stream`, then reports NEXUS_ETIMEOUT if any kernel of this
+ * library on the current device gave up a bounded wait since the last call
+ * (and clears that record), NEXUS_ECUDA if the stream reports an error,
+ * else NEXUS_OK. */
+nexus_status nexus_device_status(nexus_stream stream);
+
+/* ---------------------------------------------------------------- policy */
+/* R(n_past) of Eq. 2 (Sec. III-C) as an exact fraction *num / *den in percent,
+ * clamped to 100. Returns NEXUS_EINVAL for K < 2, M < 1 or R_base outside [0, 100]. */
+nexus_status nexus_recompute_pct(int32_t n_past, const nexus_policy* policy,
+                                 int64_t* num, int64_t* den);
+
+/* ceil(S * R(n_past) / 100), at most S: the suffix that is invalidated and
+ * re-decoded after a splice (Sec. V-A). Negative on invalid input. */
+int32_t nexus_redecode_len(int32_t S, int32_t n_past, const nexus_policy* policy);
+
+/* ceil(S * pct / 100) for a fixed percentage in [0, 100]; negative on invalid input. */
+int32_t nexus_suffix_len(int32_t S, int32_t pct);
+
+/* Fail-closed gate of Sec. III-B / III-C: NEXUS_EDECLINED if n_past exceeds the
+ * threshold P and fewer than nexus_redecode_len(S, n_past) rows will be
+ * re-decoded, else NEXUS_OK. */
+nexus_status nexus_check_splice(int32_t n_past, int32_t S, int32_t n_redecode,
+                                const nexus_policy* policy);
+
+/* ------------------------------------------------------------- page pool */
+/* Host allocator of cache pages (the analogue of the paper's cache-line
+ * hardened bitmap allocator, Sec. V-C). `order` (nullable) gives the order in
+ * which pages are handed out; NULL means 0, 1, 2, ... Thread-safe. */
+nexus_status nexus_page_pool_create(int64_t n_pages, const int32_t* order,
+                                    nexus_page_pool** out);
+void nexus_page_pool_destroy(nexus_page_pool* pool);
+/* Takes n pages in pool order; NEXUS_ENOMEM (and no change) if fewer are free. */
+nexus_status nexus_page_pool_alloc(nexus_page_pool* pool, int32_t n, int32_t* pages);
+/* Returns pages to the back of the order; NEXUS_ERANGE for an id outside the
+ * pool, NEXUS_EINVAL for a page that is already free (nothing is freed then). */
+nexus_status nexus_page_pool_free(nexus_page_pool* pool, int32_t n, const int32_t* pages);
+int64_t nexus_page_pool_available(const nexus_page_pool* pool);
+
+/* --------------------------------------------------------------- planner */
+/* Plans the insertion of blocks into one sequence of length n_past whose page
+ * table is h_old_pt (host, [max_pages]). The post-splice sequence is
+ * live[0:d1] ++ block1 ++ live[d1:d2] ++ ... ++ live[dk:n_past]; block rows are
+ * reanchored by delta = final position - base_pos (Sec. III-B) and displaced
+ * live rows are re-rotated by the number of block rows inserted before them.
+ * Pages that hold no changed row are shared with the old table; every other
+ * page of the new table is taken from `pool`, so no destination row overlaps a
+ * source row. Appending at the cursor (all depths == n_past) keeps the
+ * partially filled last page in place.
+ *   h_new_pt    out [max_pages]: the new page table (entries past the
+ *               sequence end are set to -1)
+ *   segs        out: the segments for nexus_splice_kv, reading live rows from
+ *               page-table row old_row and writing row new_row
+ *   freed       out (nullable, capacity max_pages): old pages the new table
+ *               no longer uses; the caller frees them once the splice is done
+ * Returns NEXUS_ENOMEM if the pool or seg_capacity is too small (the pool is
+ * then unchanged), NEXUS_ERANGE if the result exceeds max_pages * 16 rows. */
+nexus_status nexus_plan_splice(nexus_page_pool* pool, const int32_t* h_old_pt,
+                               int32_t n_past, int32_t max_pages,
+                               const nexus_block* blocks, int32_t n_blocks,
+                               const nexus_insert* inserts, int32_t n_inserts,
+                               int32_t old_row, int32_t new_row, int32_t* h_new_pt,
+                               nexus_splice_segment* segs, int32_t seg_capacity,
+                               int32_t* n_segs, int32_t* freed, int32_t* n_freed);
+
+/* ----------------------------------------------------------------- splice */
+/* Writes every segment for layers [layer_begin, layer_end) in one launch
+ * (Sec. V-A splice; Sec. III-B reanchoring; Sec. V-B transposed V). K rows are
+ * rotated by the segment's delta in float32 from float64-reduced angles and
+ * stored round-to-nearest-even; delta = 0 copies K bits unchanged; V bits are
+ * always copied unchanged.
+ *   d_page_tables  device int32 [n_rows][max_pages]
+ *   h_page_tables  host copy of the same (nullable). When given, every page
+ *                  id is range-checked and destination rows are checked not
+ *                  to overlap each other or any source row (NEXUS_EOVERLAP);
+ *                  a segment may read and write the same rows only if it is
+ *                  K-only (an in-place rotation).
+ *   blocks         host array of n_blocks descriptors; each block's RoPE
+ *                  parameters and shape must match the cache
+ *                  (NEXUS_EROPE_MISMATCH / NEXUS_ELAYOUT)
+ *   segments       host array of n_segments (at most 4096)
+ * Block layer l feeds cache layer l. */
+nexus_status nexus_splice_kv(const nexus_kv_cache* cache,
+                             const int32_t* d_page_tables, const int32_t* h_page_tables,
+                             int32_t n_rows, int32_t max_pages,
+                             const nexus_block* blocks, int32_t n_blocks,
+                             const nexus_splice_segment* segments, int32_t n_segments,
+                             int32_t layer_begin, int32_t layer_end, nexus_stream stream);
+
+/* In-place rotation of the keys of positions [pos_begin, pos_begin + n_tokens)
+ * of page-table row `row` by `delta` positions (Sec. III-B, Eq. 1), for layers
+ * [layer_begin, layer_end). V is untouched. */
+nexus_status nexus_rope_rerotate(const nexus_kv_cache* cache,
+                                 const int32_t* d_page_tables, const int32_t* h_page_tables,
+                                 int32_t n_rows, int32_t max_pages, int32_t row,
+                                 int32_t pos_begin, int32_t n_tokens, int32_t delta,
+                                 int32_t layer_begin, int32_t layer_end, nexus_stream stream);
+
+/* The rotation of nexus_rope_rerotate written, unrounded, as float32 into
+ * out_f32 (device [layer_end - layer_begin][n_tokens][n_kv_heads][head_dim]);
+ * the cache is only read. It exposes the float32 arithmetic ahead of the bf16
+ * store for verification. */
+nexus_status nexus_rope_rerotate_f32(const nexus_kv_cache* cache,
+                                     const int32_t* d_page_tables, const int32_t* h_page_tables,
+                                     int32_t n_rows, int32_t max_pages, int32_t row,
+                                     int32_t pos_begin, int32_t n_tokens, int32_t delta,
+                                     int32_t layer_begin, int32_t layer_end,
+                                     float* out_f32, nexus_stream stream);
+
+/* Bit-exact copy of whole pages src_pages[i] -> dst_pages[i] (K and V, all
+ * heads) for layers [layer_begin, layer_end): the in-arena KV copy of the
+ * paper's L0 radix arena (Sec. V-D), also used for copy-on-write. Host arrays,
+ * at most 2048 pairs per call; NEXUS_EOVERLAP if a page is both a source and a
+ * destination or is written twice. */
+nexus_status nexus_copy_pages(const nexus_kv_cache* cache, const int32_t* h_src_pages,
+                              const int32_t* h_dst_pages, int32_t n, int32_t layer_begin,
+                              int32_t layer_end, nexus_stream stream);
+
+/* -------------------------------------------------------------- attention */
+/* Causal GQA attention of the last q_len[s] positions of each sequence s over
+ * its kv_len[s] cached positions (Sec. III-A; the redecoded suffix of
+ * Sec. III-C / Sec. V-A). Query t of sequence s sits at position
+ * kv_len[s] - q_len[s] + t and sees keys at positions <= its own; query head h
+ * reads KV head h / (n_q_heads / n_kv_heads). Scores are scaled by
+ * 1/sqrt(head_dim). bf16 operands, float32 accumulation; O is bf16 and LSE
+ * (natural log of the softmax denominator of the scaled scores) float32.
+ *   d_page_tables  device int32 [n_rows][max_pages]
+ *   h_rows         host [n_seqs]: page-table row of each sequence (nullable:
+ *                  sequence s uses row s)
+ *   h_kv_len, h_q_len  host [n_seqs]; 0 <= q_len <= kv_len <= max_pages * 16
+ *   q, out         device bf16, see the layout above; sequences are packed
+ *                  back to back along the token axis in order
+ *   lse            device float (nullable)
+ *   n_seqs         1 .. 512
+ *   split_kv       number of key-range partitions: 1 = none, 0 = chosen by
+ *                  the library from the work size and SM count, up to 64
+ *   workspace      device scratch for split partials (nullable when no split
+ *                  is used); its size comes from nexus_attention_workspace_size
+ *                  with the same arguments; NEXUS_ENOMEM if too small
+ * Cache slots past kv_len may hold any bits: they never reach the output. */
+nexus_status nexus_suffix_attention(const nexus_kv_cache* cache,
+                                    const int32_t* d_page_tables, int32_t n_rows,
+                                    int32_t max_pages, int32_t n_seqs, const int32_t* h_rows,
+                                    const int32_t* h_kv_len, const int32_t* h_q_len,
+                                    const void* q, void* out, float* lse, int32_t n_q_heads,
+                                    int32_t layer_begin, int32_t layer_end, int32_t split_kv,
+                                    void* workspace, size_t workspace_bytes,
+                                    nexus_stream stream);
+
+/* Full causal re-prefill: nexus_suffix_attention with q_len = kv_len (the
+ * R = 100 % end point of Eq. 2, Sec. III-C). */
+nexus_status nexus_reprefill(const nexus_kv_cache* cache, const int32_t* d_page_tables,
+                             int32_t n_rows, int32_t max_pages, int32_t n_seqs,
+                             const int32_t* h_rows, const int32_t* h_kv_len, const void* q,
+                             void* out, float* lse, int32_t n_q_heads, int32_t layer_begin,
+                             int32_t layer_end, int32_t split_kv, void* workspace,
+                             size_t workspace_bytes, nexus_stream stream);
+
+/* Bytes of workspace nexus_suffix_attention needs for these arguments
+ * (0 when no split is used). *splits_out (nullable) receives the partition
+ * count the call will use. Uses the current device's SM count, or 152 when no
+ * device is visible. */
+size_t nexus_attention_workspace_size(int32_t n_seqs, const int32_t* h_kv_len,
+                                      const int32_t* h_q_len, int32_t n_q_heads,
+                                      int32_t n_kv_heads, int32_t n_layers_call,
+                                      int32_t split_kv, int32_t* splits_out);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* NEXUS_H */

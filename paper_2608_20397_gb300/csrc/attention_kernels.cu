@@ -1,0 +1,525 @@
+// Causal GQA suffix-redecode / re-prefill attention on sm_103a tensor cores
+// (softmax(QK^T / sqrt(d)) V of Sec. III-A over the redecoded suffix of
+// Sec. III-C / Sec. V-A), plus the split-KV partial merge.
+//
+// One CTA owns one 128-row query tile of one KV head: rows are (token, head in
+// the GQA group) pairs, 128 / group tokens x group heads, so every K/V tile
+// brought into shared memory serves all query heads that read it. Per CTA:
+//
+//   warp 4    TMA producer: the Q tile once, then K and V tiles of 128 keys
+//             (eight 16-token pages each, fetched through the page table)
+//             into a two-stage ring
+//   warp 5    MMA issuer: S = Q K^T into TMEM (double-buffered), then
+//             O += P V into TMEM, with tcgen05.mma (bf16 in, f32 accumulate)
+//   warps 0-3 softmax: thread i owns TMEM lane i (= tile row i); online
+//             softmax in the log2 domain with a lazily moved running max,
+//             P written to shared memory as bf16, final O / l and LSE
+//
+// TMEM columns: S0 [0,128), S1 [128,256), O [256,384) of a 512-column
+// allocation. Every wait is bounded; on expiry the CTA records a timeout,
+// drains its in-flight copies and MMAs, frees TMEM and exits.
+#include <cuda_bf16.h>
+
+#include "internal.h"
+#include "ptx.cuh"
+
+namespace nexus {
+
+__device__ unsigned int g_attn_timeout = 0;
+
+namespace {
+using namespace ptx;
+
+constexpr int BM = 128;   // query rows per tile
+constexpr int BN = 128;   // keys per tile
+constexpr int D = kHeadDim;
+constexpr int kStages = 2;
+constexpr int kThreads = 192;
+constexpr int kProducerWarp = 4;
+constexpr int kMmaWarp = 5;
+constexpr uint32_t kTileBytes = BM * D * 2;   // 32 KiB
+constexpr uint32_t kHalf = 16384;             // one 64-column half of a tile
+constexpr uint64_t kBudgetNs = 2000000000ull; // 2 s per wait
+constexpr uint64_t kDrainNs = 200000000ull;   // 0.2 s to drain after an abort
+constexpr float kRescaleThreshold = 8.0f;     // move the running max only past 2^8 growth
+
+constexpr uint32_t OFF_Q = 0;
+constexpr uint32_t OFF_K = OFF_Q + kTileBytes;
+constexpr uint32_t OFF_V = OFF_K + kStages * kTileBytes;
+constexpr uint32_t OFF_P = OFF_V + kStages * kTileBytes;
+constexpr uint32_t OFF_BAR = OFF_P + kTileBytes;
+enum {
+  B_Q = 0,
+  B_KF = 1,      // +stage
+  B_VF = 3,      // +stage
+  B_KVE = 5,     // +stage
+  B_SF = 7,      // +buffer
+  B_SFREE = 9,   // +buffer
+  B_PF = 11,
+  B_OD = 12,
+  B_FIN = 13,
+  kNumBars = 14
+};
+constexpr uint32_t OFF_MISC = OFF_BAR + kNumBars * 8;
+constexpr uint32_t kSmemUsed = OFF_MISC + 16;
+constexpr uint32_t kSmemBytes = kSmemUsed + 1024;   // slack for 1024-byte alignment
+
+constexpr uint32_t TM_S0 = 0, TM_O = 256;
+
+__device__ __forceinline__ void record_timeout(volatile int* abort) {
+  *abort = 1;
+  atomicOr(&g_attn_timeout, 1u);
+}
+
+struct Tile {
+  int seq, qt, kv, layer_rel, split;
+  int tok0, ntok, pos0, kt_begin, n_tiles;
+};
+
+__device__ __forceinline__ Tile decode_tile(const AttnLaunch& p) {
+  Tile t;
+  const int rev = p.total_tiles - 1 - (int)blockIdx.x;   // deepest query tiles first
+  int lo = 0, hi = p.n_seqs - 1;
+  while (lo < hi) {
+    const int mid = (lo + hi + 1) >> 1;
+    if (p.tile_prefix[mid] <= rev) lo = mid; else hi = mid - 1;
+  }
+  t.seq = lo;
+  t.qt = rev - p.tile_prefix[lo];
+  t.kv = blockIdx.y;
+  t.layer_rel = blockIdx.z / p.splits;
+  t.split = blockIdx.z % p.splits;
+  const AttnSeq& s = p.seq[lo];
+  t.tok0 = t.qt * p.tile_tokens;
+  t.ntok = min(p.tile_tokens, s.q_len - t.tok0);
+  t.pos0 = s.kv_len - s.q_len + t.tok0;
+  const int pos_last = t.pos0 + t.ntok - 1;
+  const int kt_total = pos_last / BN + 1;
+  const int per = (kt_total + p.splits - 1) / p.splits;
+  t.kt_begin = t.split * per;
+  t.n_tiles = max(0, min(kt_total, t.kt_begin + per) - t.kt_begin);
+  return t;
+}
+
+// Zeroes V rows of keys [r0, 128) of one stage, so cache slots past kv_len
+// (whatever bits they hold) contribute exactly 0 to P V.
+__device__ __forceinline__ void zero_v_rows(uint8_t* vbuf, int r0, bool vt, int lane) {
+  if (!vt) {
+    // two halves of [128 keys][128 B]
+    for (int i = lane; i < 2 * (BN - r0) * 8; i += 32) {
+      const int half = i / ((BN - r0) * 8);
+      const int rem = i % ((BN - r0) * 8);
+      const int row = r0 + rem / 8;
+      reinterpret_cast<uint4*>(vbuf + half * kHalf + row * 128)[rem % 8] = make_uint4(0, 0, 0, 0);
+    }
+  } else {
+    // eight pages of [128 d][16 keys] with the 32-byte swizzle (16-byte chunk
+    // index XOR bit 2 of the row)
+    for (int i = lane; i < 8 * D; i += 32) {
+      const int pg = i / D, d = i % D;
+      const int k0 = pg * 16;
+      if (k0 + 16 <= r0) continue;
+      uint16_t* row = reinterpret_cast<uint16_t*>(vbuf + pg * 4096 + d * 32);
+      for (int s = max(0, r0 - k0); s < 16; ++s) {
+        const int chunk = (s >> 3) ^ ((d >> 2) & 1);
+        row[chunk * 8 + (s & 7)] = 0;
+      }
+    }
+  }
+}
+
+__global__ void __launch_bounds__(kThreads, 1)
+attention_kernel(const __grid_constant__ AttnLaunch p, const __grid_constant__ AttnMaps maps) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~static_cast<uintptr_t>(1023));
+  const uint32_t sbase = smem_u32(smem);
+  auto bar = [&](int i) -> uint32_t { return sbase + OFF_BAR + 8u * i; };
+  volatile uint32_t* tmem_slot = reinterpret_cast<volatile uint32_t*>(smem + OFF_MISC);
+  volatile int* abort = reinterpret_cast<volatile int*>(smem + OFF_MISC + 4);
+  volatile int* never = reinterpret_cast<volatile int*>(smem + OFF_MISC + 8);   // stays 0
+  const volatile unsigned int* gabort = &g_attn_timeout;
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  const Tile t = decode_tile(p);
+  const AttnSeq sq = p.seq[t.seq];
+  const int G = p.group;
+  const int layer = p.layer_begin + t.layer_rel;
+
+  // ---- setup: zero the Q rows no TMA box writes, init barriers, alloc TMEM
+  {
+    const int rows_loaded = G * p.tile_tokens;
+    for (int i = threadIdx.x; i < 2 * (BM - rows_loaded) * 8; i += kThreads) {
+      const int half = i / ((BM - rows_loaded) * 8);
+      const int rem = i % ((BM - rows_loaded) * 8);
+      reinterpret_cast<uint4*>(smem + OFF_Q + half * kHalf + (rows_loaded + rem / 8) * 128)[rem % 8] =
+          make_uint4(0, 0, 0, 0);
+    }
+    fence_proxy_async_smem();
+  }
+  if (threadIdx.x == 0) {
+    mbar_init(bar(B_Q), 1);
+    for (int s = 0; s < kStages; ++s) {
+      mbar_init(bar(B_KF + s), 1);
+      mbar_init(bar(B_VF + s), 1);
+      mbar_init(bar(B_KVE + s), 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(bar(B_SF + b), 1);
+      mbar_init(bar(B_SFREE + b), 128);
+    }
+    mbar_init(bar(B_PF), 128);
+    mbar_init(bar(B_OD), 1);
+    mbar_init(bar(B_FIN), 1);
+    *abort = 0;
+    *never = 0;
+    fence_mbar_init();
+  }
+  if (warp == kMmaWarp) {
+    tmem_alloc(sbase + OFF_MISC, 512);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  const bool vt = p.v_transposed != 0;
+  const int n_tiles = t.n_tiles;
+
+  if (warp == kProducerWarp) {
+    // ------------------------------------------------------ TMA producer
+    const int32_t* pt = p.page_tables + (int64_t)sq.pt_row * p.max_pages;
+    const int pg_max = (sq.kv_len - 1) / kPageSize;
+    int issued = 0;
+    if (n_tiles > 0) {
+      if (lane == 0) {
+        prefetch_tmap(&maps.q);
+        prefetch_tmap(&maps.k);
+        prefetch_tmap(&maps.v);
+        mbar_arrive_expect_tx(bar(B_Q), 2u * G * p.tile_tokens * 128u);
+        for (int half = 0; half < 2; ++half)
+          tma_load_4d(sbase + OFF_Q + half * kHalf, &maps.q, bar(B_Q), half * 64, t.kv * G,
+                      sq.q_off + t.tok0, t.layer_rel);
+      }
+      for (int it = 0; it < n_tiles; ++it) {
+        const int st = it & 1;
+        if (it >= 2) {
+          bool ok = mbar_wait(bar(B_KVE + st), ((it >> 1) - 1) & 1, kBudgetNs, abort, gabort);
+          ok = __all_sync(0xffffffffu, ok);
+          if (!ok) { if (lane == 0) record_timeout(abort); break; }
+        }
+        const int kt = t.kt_begin + it;
+        int page = 0;
+        if (lane < 8) page = pt[min(kt * 8 + lane, pg_max)];
+        if (lane == 0) {
+          mbar_arrive_expect_tx(bar(B_KF + st), kTileBytes);
+          mbar_arrive_expect_tx(bar(B_VF + st), kTileBytes);
+        }
+        __syncwarp();
+        if (lane < 8) {
+          const int gp = layer * p.n_pages + page;
+          const uint32_t kdst = sbase + OFF_K + st * kTileBytes + lane * 2048;
+          const uint32_t vdst = sbase + OFF_V + st * kTileBytes;
+          tma_load_4d(kdst, &maps.k, bar(B_KF + st), 0, 0, t.kv, gp);
+          tma_load_4d(kdst + kHalf, &maps.k, bar(B_KF + st), 64, 0, t.kv, gp);
+          if (!vt) {
+            tma_load_4d(vdst + lane * 2048, &maps.v, bar(B_VF + st), 0, 0, t.kv, gp);
+            tma_load_4d(vdst + lane * 2048 + kHalf, &maps.v, bar(B_VF + st), 64, 0, t.kv, gp);
+          } else {
+            tma_load_4d(vdst + lane * 4096, &maps.v, bar(B_VF + st), 0, 0, t.kv, gp);
+          }
+        }
+        issued = it + 1;
+      }
+      if (*abort) {
+        // Let the copies still in flight land before the CTA exits.
+        for (int it = max(0, issued - 2); it < issued; ++it) {
+          const int st = it & 1;
+          mbar_wait(bar(B_KF + st), (it >> 1) & 1, kDrainNs, never);
+          mbar_wait(bar(B_VF + st), (it >> 1) & 1, kDrainNs, never);
+        }
+      }
+    }
+  } else if (warp == kMmaWarp) {
+    // ------------------------------------------------------ MMA issuer
+    constexpr uint32_t idesc_qk = idesc_bf16_f32(BM, BN, false);
+    const uint32_t idesc_pv = idesc_bf16_f32(BM, D, !vt);
+    bool ok = true;
+    if (n_tiles > 0) {
+      ok = mbar_wait(bar(B_Q), 0, kBudgetNs, abort, gabort);
+      ok = __all_sync(0xffffffffu, ok);
+      for (int it = 0; ok && it <= n_tiles; ++it) {
+        if (it < n_tiles) {
+          const int st = it & 1;
+          bool w = mbar_wait(bar(B_KF + st), (it >> 1) & 1, kBudgetNs, abort, gabort);
+          if (w && it >= 2) w = mbar_wait(bar(B_SFREE + st), ((it >> 1) - 1) & 1, kBudgetNs, abort, gabort);
+          ok = __all_sync(0xffffffffu, w);
+          if (!ok) break;
+          tc_fence_after();
+          if (lane == 0) {
+            const uint32_t qa = sbase + OFF_Q;
+            const uint32_t ka = sbase + OFF_K + st * kTileBytes;
+#pragma unroll
+            for (int kk = 0; kk < D / 16; ++kk) {
+              const uint32_t off = (kk >> 2) * kHalf + (kk & 3) * 32;
+              mma_bf16(tmem + TM_S0 + st * 128, smem_desc(qa + off, 16, 1024, kSwizzle128B),
+                       smem_desc(ka + off, 16, 1024, kSwizzle128B), idesc_qk, kk > 0);
+            }
+            mma_commit(bar(B_SF + st));
+          }
+          __syncwarp();
+        }
+        if (it >= 1) {
+          const int j = it - 1;
+          const int st = j & 1;
+          bool w = mbar_wait(bar(B_PF), j & 1, kBudgetNs, abort, gabort);
+          if (w) w = mbar_wait(bar(B_VF + st), (j >> 1) & 1, kBudgetNs, abort, gabort);
+          ok = __all_sync(0xffffffffu, w);
+          if (!ok) break;
+          const int key0 = (t.kt_begin + j) * BN;
+          if (key0 + BN > sq.kv_len) {
+            zero_v_rows(smem + OFF_V + st * kTileBytes, sq.kv_len - key0, vt, lane);
+            fence_proxy_async_smem();
+            __syncwarp();
+          }
+          tc_fence_after();
+          if (lane == 0) {
+            const uint32_t pa = sbase + OFF_P;
+            const uint32_t va = sbase + OFF_V + st * kTileBytes;
+#pragma unroll
+            for (int kk = 0; kk < BN / 16; ++kk) {
+              const uint64_t adesc =
+                  smem_desc(pa + (kk >> 2) * kHalf + (kk & 3) * 32, 16, 1024, kSwizzle128B);
+              // row-major V: MN-major, 64-wide d halves 16 KiB apart (LBO), 8-key
+              // groups 1 KiB apart (SBO); token-innermost V: K-major pages of
+              // [128 d][16 keys], 8-row groups 256 B apart.
+              const uint64_t bdesc = vt ? smem_desc(va + kk * 4096, 16, 256, kSwizzle32B)
+                                        : smem_desc(va + kk * 2048, kHalf, 1024, kSwizzle128B);
+              mma_bf16(tmem + TM_O, adesc, bdesc, idesc_pv, (j > 0 || kk > 0) ? 1u : 0u);
+            }
+            mma_commit(bar(B_OD));
+            mma_commit(bar(B_KVE + st));
+          }
+          __syncwarp();
+        }
+      }
+      if (!ok && lane == 0) record_timeout(abort);
+    }
+    // Every MMA this thread issued has finished before TMEM is released.
+    if (n_tiles > 0) {
+      if (lane == 0) mma_commit(bar(B_FIN));
+      __syncwarp();
+      mbar_wait(bar(B_FIN), 0, kDrainNs, never);
+    }
+  } else {
+    // ------------------------------------------------------ softmax warps
+    const int r = threadIdx.x;                 // tile row == TMEM lane
+    const uint32_t lane_base = static_cast<uint32_t>(warp * 32) << 16;
+    const int tr = r / G;                      // token within the tile
+    const int pos_r = t.pos0 + tr;
+    const bool row_valid = (r < G * p.tile_tokens) && (tr < t.ntok);
+    float m_run = -INFINITY;
+    float l_run = 0.f;
+    bool ok = true;
+    for (int it = 0; it < n_tiles; ++it) {
+      const int sb = it & 1;
+      bool w = mbar_wait(bar(B_SF + sb), (it >> 1) & 1, kBudgetNs, abort, gabort);
+      ok = __all_sync(0xffffffffu, w);
+      if (!ok) break;
+      tc_fence_after();
+      float s[BN];
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        uint32_t v[32];
+        tmem_ld32(tmem + lane_base + TM_S0 + sb * 128 + q * 32, v);
+        tmem_ld_wait();
+#pragma unroll
+        for (int e = 0; e < 32; ++e) s[q * 32 + e] = __uint_as_float(v[e]);
+      }
+      tc_fence_before();
+      mbar_arrive(bar(B_SFREE + sb));
+
+      const int lim = pos_r - (t.kt_begin + it) * BN;   // keys j <= lim are visible
+      float mx = -INFINITY;
+      if (lim >= BN - 1) {
+#pragma unroll
+        for (int j = 0; j < BN; ++j) { s[j] *= p.scale_log2; mx = fmaxf(mx, s[j]); }
+      } else {
+#pragma unroll
+        for (int j = 0; j < BN; ++j) {
+          s[j] = (j <= lim) ? s[j] * p.scale_log2 : -INFINITY;
+          mx = fmaxf(mx, s[j]);
+        }
+      }
+      // Move the running max only when the new one is far above it; the
+      // stale max keeps every p <= 2^8 and O / l unchanged.
+      float alpha = 1.f;
+      bool rescale = false;
+      if (mx > -INFINITY && (m_run == -INFINITY || mx > m_run + kRescaleThreshold)) {
+        if (m_run != -INFINITY) { alpha = ex2_approx(m_run - mx); rescale = true; }
+        m_run = mx;
+      }
+      const float m_use = (m_run == -INFINITY) ? 0.f : m_run;
+      uint32_t pk[BN / 2];
+      float sum = 0.f;
+#pragma unroll
+      for (int j = 0; j < BN; j += 2) {
+        const float p0 = ex2_approx(s[j] - m_use);
+        const float p1 = ex2_approx(s[j + 1] - m_use);
+        sum += p0 + p1;
+        pk[j / 2] = pack_bf16x2(p0, p1);
+      }
+      l_run = l_run * alpha + sum;
+
+      if (it >= 1) {
+        // PV of the previous tile must be done before O is rescaled and P reused.
+        w = mbar_wait(bar(B_OD), (it - 1) & 1, kBudgetNs, abort, gabort);
+        ok = __all_sync(0xffffffffu, w);
+        if (!ok) break;
+        tc_fence_after();
+        if (__any_sync(0xffffffffu, rescale)) {
+#pragma unroll
+          for (int q = 0; q < 4; ++q) {
+            uint32_t v[32];
+            tmem_ld32(tmem + lane_base + TM_O + q * 32, v);
+            tmem_ld_wait();
+#pragma unroll
+            for (int e = 0; e < 32; ++e) v[e] = __float_as_uint(__uint_as_float(v[e]) * alpha);
+            tmem_st32(tmem + lane_base + TM_O + q * 32, v);
+          }
+          tmem_st_wait();
+        }
+      }
+      // P row -> shared memory, K-major with the 128-byte swizzle.
+      const uint32_t prow = sbase + OFF_P + r * 128;
+#pragma unroll
+      for (int c = 0; c < BN / 8; ++c) {
+        const uint32_t addr = prow + (c >> 3) * kHalf + (((c & 7) ^ (r & 7)) << 4);
+        st_shared_v4(addr, pk[c * 4], pk[c * 4 + 1], pk[c * 4 + 2], pk[c * 4 + 3]);
+      }
+      fence_proxy_async_smem();
+      tc_fence_before();
+      mbar_arrive(bar(B_PF));
+    }
+    if (!ok && r == 0) record_timeout(abort);
+
+    // ---- epilogue: O / l and LSE
+    float o[D];
+    bool have_o = false;
+    if (ok && n_tiles > 0) {
+      bool w = mbar_wait(bar(B_OD), (n_tiles - 1) & 1, kBudgetNs, abort, gabort);
+      w = __all_sync(0xffffffffu, w);
+      if (w) {
+        tc_fence_after();
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          uint32_t v[32];
+          tmem_ld32(tmem + lane_base + TM_O + q * 32, v);
+          tmem_ld_wait();
+#pragma unroll
+          for (int e = 0; e < 32; ++e) o[q * 32 + e] = __uint_as_float(v[e]);
+        }
+        have_o = true;
+      } else if (r == 0) {
+        record_timeout(abort);
+      }
+    }
+    if (row_valid) {
+      const float inv_l = (have_o && l_run > 0.f) ? 1.f / l_run : 0.f;
+      const float lse = (have_o && l_run > 0.f) ? (m_run + log2f(l_run)) * 0.69314718055994531f
+                                               : -INFINITY;
+      const int tok = sq.q_off + t.tok0 + tr;
+      const int head = t.kv * G + (r % G);
+      const int64_t row = ((int64_t)t.layer_rel * p.n_tok + tok) * p.n_q_heads + head;
+      if (p.splits == 1) {
+        uint4* dst = reinterpret_cast<uint4*>(p.out + row * D);
+#pragma unroll
+        for (int c = 0; c < D / 8; ++c) {
+          float v[8];
+#pragma unroll
+          for (int e = 0; e < 8; ++e) v[e] = have_o ? o[c * 8 + e] * inv_l : 0.f;
+          dst[c] = make_uint4(pack_bf16x2(v[0], v[1]), pack_bf16x2(v[2], v[3]),
+                              pack_bf16x2(v[4], v[5]), pack_bf16x2(v[6], v[7]));
+        }
+        if (p.lse) p.lse[row] = lse;
+      } else {
+        const int64_t rows_per_split = (int64_t)p.n_layers_call * p.n_tok * p.n_q_heads;
+        float4* dst = reinterpret_cast<float4*>(p.part_o + ((int64_t)t.split * rows_per_split + row) * D);
+#pragma unroll
+        for (int c = 0; c < D / 4; ++c)
+          dst[c] = have_o ? make_float4(o[4 * c] * inv_l, o[4 * c + 1] * inv_l,
+                                        o[4 * c + 2] * inv_l, o[4 * c + 3] * inv_l)
+                          : make_float4(0.f, 0.f, 0.f, 0.f);
+        p.part_lse[(int64_t)t.split * rows_per_split + row] = lse;
+      }
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  if (warp == kMmaWarp) tmem_dealloc(tmem, 512);
+}
+
+// Merge of split-KV partials: one warp per (layer, token, head) row. Lane s
+// holds split s's LSE; the max and the weight sum are warp-shuffle
+// reductions, then every lane accumulates its four columns over the splits.
+__global__ void __launch_bounds__(128) combine_kernel(const __grid_constant__ AttnLaunch p) {
+  const int64_t rows = (int64_t)p.n_layers_call * p.n_tok * p.n_q_heads;
+  const int64_t row = (int64_t)blockIdx.x * 4 + (threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31;
+  if (row >= rows) return;
+  const float l_s = lane < p.splits ? p.part_lse[(int64_t)lane * rows + row] : -INFINITY;
+  float mx = l_s;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+  const float w = (mx == -INFINITY || l_s == -INFINITY) ? 0.f : expf(l_s - mx);
+  float wsum = w;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) wsum += __shfl_xor_sync(0xffffffffu, wsum, o);
+  float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+  for (int s = 0; s < p.splits; ++s) {
+    const float ws = __shfl_sync(0xffffffffu, w, s);
+    if (ws == 0.f) continue;
+    const float4 v = reinterpret_cast<const float4*>(p.part_o + ((int64_t)s * rows + row) * D)[lane];
+    acc.x += ws * v.x; acc.y += ws * v.y; acc.z += ws * v.z; acc.w += ws * v.w;
+  }
+  const float inv = wsum > 0.f ? 1.f / wsum : 0.f;
+  uint2 outv = make_uint2(pack_bf16x2(acc.x * inv, acc.y * inv), pack_bf16x2(acc.z * inv, acc.w * inv));
+  reinterpret_cast<uint2*>(p.out + row * D)[lane] = outv;
+  if (p.lse && lane == 0) p.lse[row] = wsum > 0.f ? mx + logf(wsum) : -INFINITY;
+}
+
+}  // namespace
+
+cudaError_t launch_attention(const AttnLaunch& p, const AttnMaps& maps, cudaStream_t stream) {
+  if (p.total_tiles <= 0 || p.n_layers_call <= 0) return cudaSuccess;
+  static_assert(kSmemBytes <= 227 * 1024, "shared memory budget");
+  cudaError_t e = cudaFuncSetAttribute(attention_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       (int)kSmemBytes);
+  if (e != cudaSuccess) return e;
+  const dim3 grid((unsigned)p.total_tiles, (unsigned)p.n_kv_heads,
+                  (unsigned)(p.n_layers_call * p.splits));
+  attention_kernel<<<grid, kThreads, kSmemBytes, stream>>>(p, maps);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_attn_combine(const AttnLaunch& p, cudaStream_t stream) {
+  const int64_t rows = (int64_t)p.n_layers_call * p.n_tok * p.n_q_heads;
+  if (rows <= 0) return cudaSuccess;
+  combine_kernel<<<(unsigned)((rows + 3) / 4), 128, 0, stream>>>(p);
+  return cudaGetLastError();
+}
+
+cudaError_t attention_take_timeout(unsigned int* flag, cudaStream_t stream) {
+  cudaError_t e = cudaStreamSynchronize(stream);
+  if (e != cudaSuccess) return e;
+  e = cudaMemcpyFromSymbol(flag, g_attn_timeout, sizeof(unsigned int));
+  if (e != cudaSuccess) return e;
+  const unsigned int zero = 0;
+  return cudaMemcpyToSymbol(g_attn_timeout, &zero, sizeof(unsigned int));
+}
+
+}  // namespace nexus

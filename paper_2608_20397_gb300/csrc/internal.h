@@ -1,0 +1,119 @@
+// Launch-side structures shared by the C-ABI layer and the CUDA kernels.
+#pragma once
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <cstdint>
+
+#include "nexus.h"
+
+namespace nexus {
+
+constexpr int kHeadDim = 128;
+constexpr int kPageSize = 16;
+constexpr int kMaxKvHeads = 16;
+
+// ------------------------------------------------------------------ splice
+// One destination run, resolved for the device. A CTA handles the rows of one
+// segment that fall into one destination page ("piece"), for one layer.
+struct DevSegment {
+  const uint16_t* src_k;     // block K at layer 0 (nullptr: source is the cache)
+  const uint16_t* src_v;     // block V at layer 0
+  int64_t src_layer_stride;  // elements between consecutive layers of the block
+  int32_t src_row;           // page-table row of a cache source (-1 for a block)
+  int32_t src_start;
+  int32_t dst_row;
+  int32_t dst_start;
+  int32_t n_tokens;
+  int32_t delta;
+  int32_t flags;
+  int32_t piece_begin;       // prefix sum of pieces over earlier segments
+};
+
+constexpr int kMaxSegmentsPerLaunch = 224;
+
+enum SpliceOut : int32_t { kOutPool = 0, kOutF32 = 1 };
+
+struct SpliceLaunch {
+  uint16_t* k_pool;
+  uint16_t* v_pool;
+  const int32_t* page_tables;
+  float* out_f32;            // kOutF32: [n_layers_call][n_tokens][Hkv][128]
+  int64_t n_pages;
+  int32_t n_kv_heads;
+  int32_t max_pages;
+  int32_t layer_begin;
+  int32_t n_layers_call;
+  int32_t n_segments;
+  int32_t n_pieces;
+  int32_t v_transposed;
+  int32_t rope_gptj;
+  int32_t out_mode;
+  int32_t out_pos_begin;     // kOutF32: source position of output token 0
+  double inv_freq_over_pi[kHeadDim / 2];   // theta_i / pi
+  DevSegment seg[kMaxSegmentsPerLaunch];
+};
+
+cudaError_t launch_splice(const SpliceLaunch& p, cudaStream_t stream);
+
+// -------------------------------------------------------------- page copy
+constexpr int kMaxPageCopies = 2048;
+struct PageCopyLaunch {
+  uint16_t* k_pool;
+  uint16_t* v_pool;
+  int64_t n_pages;
+  int32_t n_kv_heads;
+  int32_t layer_begin;
+  int32_t n_layers_call;
+  int32_t n;
+  int32_t src[kMaxPageCopies];
+  int32_t dst[kMaxPageCopies];
+};
+cudaError_t launch_page_copy(const PageCopyLaunch& p, cudaStream_t stream);
+
+// --------------------------------------------------------------- attention
+constexpr int kMaxSeqs = 512;
+constexpr int kMaxSplits = 32;
+
+struct AttnSeq {
+  int32_t kv_len;
+  int32_t q_len;
+  int32_t q_off;        // first packed token of this sequence in Q / O
+  int32_t pt_row;
+};
+
+struct AttnLaunch {
+  const int32_t* page_tables;
+  uint16_t* out;            // bf16 O (no split) [n_layers_call][n_tok][Hq][128]
+  float* lse;               // nullable
+  float* part_o;            // split partials [splits][n_layers_call][n_tok][Hq][128]
+  float* part_lse;          // [splits][n_layers_call][n_tok][Hq]
+  int32_t max_pages;
+  int32_t n_q_heads;
+  int32_t n_kv_heads;
+  int32_t group;            // n_q_heads / n_kv_heads
+  int32_t tile_tokens;      // query tokens per 128-row tile = 128 / group
+  int32_t n_tok;            // packed tokens (sum of q_len)
+  int32_t n_pages;          // pages per layer (as int: the pool index range)
+  int32_t layer_begin;
+  int32_t n_layers_call;
+  int32_t n_seqs;
+  int32_t splits;
+  int32_t v_transposed;
+  int32_t total_tiles;      // sum over sequences of q tiles
+  float scale_log2;         // log2(e) / sqrt(head_dim)
+  int32_t tile_prefix[kMaxSeqs + 1];
+  AttnSeq seq[kMaxSeqs];
+};
+
+struct AttnMaps {
+  CUtensorMap q;
+  CUtensorMap k;
+  CUtensorMap v;
+};
+
+cudaError_t launch_attention(const AttnLaunch& p, const AttnMaps& maps, cudaStream_t stream);
+cudaError_t launch_attn_combine(const AttnLaunch& p, cudaStream_t stream);
+// Reads and clears the timeout record of the current device.
+cudaError_t attention_take_timeout(unsigned int* flag, cudaStream_t stream);
+
+}  // namespace nexus

@@ -1,0 +1,527 @@
+// C-ABI entry points of the device path: argument validation on the host,
+// TMA tensor-map encoding, and the launches of the splice, page-copy and
+// attention kernels.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+#include <cuda_runtime.h>
+
+#include <algorithm>
+#include <cmath>
+#include <cstring>
+#include <memory>
+#include <mutex>
+#include <vector>
+
+#include "internal.h"
+
+using namespace nexus;
+
+namespace {
+
+constexpr int kNumSmsFallback = 152;
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+nexus_status check_cache(const nexus_kv_cache* c) {
+  if (!c || !c->k_pool || !c->v_pool) return NEXUS_EINVAL;
+  if (c->head_dim != kHeadDim || c->page_size != kPageSize) return NEXUS_ELAYOUT;
+  if (c->n_kv_heads < 1 || c->n_kv_heads > kMaxKvHeads || c->n_layers < 1 || c->n_pages < 1)
+    return NEXUS_EINVAL;
+  if (c->n_pages * static_cast<int64_t>(c->n_layers) > 0x7FFFFFFFLL) return NEXUS_ERANGE;
+  if (!aligned16(c->k_pool) || !aligned16(c->v_pool)) return NEXUS_ELAYOUT;
+  if (c->rope_type != NEXUS_ROPE_NEOX && c->rope_type != NEXUS_ROPE_GPTJ) return NEXUS_EINVAL;
+  if (!(c->rope_theta > 1.0) || !(c->rope_freq_scale > 0.0) || !std::isfinite(c->rope_theta) ||
+      !std::isfinite(c->rope_freq_scale))
+    return NEXUS_EINVAL;
+  if (c->v_transposed != 0 && c->v_transposed != 1) return NEXUS_EINVAL;
+  return NEXUS_OK;
+}
+
+nexus_status check_layers(const nexus_kv_cache* c, int32_t lb, int32_t le) {
+  if (lb < 0 || le > c->n_layers || lb > le) return NEXUS_ERANGE;
+  return NEXUS_OK;
+}
+
+// A block is spliced only if its header matches the runtime model (Sec. V-A).
+nexus_status check_block(const nexus_kv_cache* c, const nexus_block& b) {
+  if (!b.k || !b.v || b.n_tokens < 0) return NEXUS_EINVAL;
+  if (!aligned16(b.k) || !aligned16(b.v)) return NEXUS_ELAYOUT;
+  if (b.n_layers != c->n_layers || b.n_kv_heads != c->n_kv_heads || b.head_dim != c->head_dim)
+    return NEXUS_ELAYOUT;
+  if (b.rope_type != c->rope_type || b.rope_theta != c->rope_theta ||
+      b.rope_freq_scale != c->rope_freq_scale)
+    return NEXUS_EROPE_MISMATCH;
+  return NEXUS_OK;
+}
+
+void fill_inv_freq_over_pi(const nexus_kv_cache* c, double* out) {
+  for (int i = 0; i < kHeadDim / 2; ++i)
+    out[i] = c->rope_freq_scale * std::pow(c->rope_theta, -2.0 * i / kHeadDim) / M_PI;
+}
+
+int num_sms() {
+  int dev = 0, n = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) { cudaGetLastError(); return kNumSmsFallback; }
+  if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0) {
+    cudaGetLastError();
+    return kNumSmsFallback;
+  }
+  return n;
+}
+
+int32_t pieces_of(int32_t dst_start, int32_t n) {
+  if (n <= 0) return 0;
+  return (dst_start + n - 1) / kPageSize - dst_start / kPageSize + 1;
+}
+
+// Destination / source slot bookkeeping for the overlap check, kept per thread
+// so repeated calls do not reallocate.
+struct SlotMarks {
+  std::vector<int32_t> owner;
+  std::vector<int64_t> touched;
+  void ensure(int64_t n) {
+    if (static_cast<int64_t>(owner.size()) < n) owner.assign(static_cast<size_t>(n), -1);
+  }
+  void reset() {
+    for (int64_t s : touched) owner[s] = -1;
+    touched.clear();
+  }
+};
+
+nexus_status validate_segments(const nexus_kv_cache* c, const int32_t* h_pt, int32_t n_rows,
+                               int32_t max_pages, const nexus_block* blocks, int32_t n_blocks,
+                               const nexus_splice_segment* segs, int32_t n_segs) {
+  const int64_t cap = static_cast<int64_t>(max_pages) * kPageSize;
+  for (int32_t i = 0; i < n_segs; ++i) {
+    const nexus_splice_segment& s = segs[i];
+    if (s.n_tokens < 0 || s.dst_start < 0 || s.src_start < 0) return NEXUS_EINVAL;
+    if (s.dst_row < 0 || s.dst_row >= n_rows) return NEXUS_ERANGE;
+    if (s.dst_start + static_cast<int64_t>(s.n_tokens) > cap) return NEXUS_ERANGE;
+    if (s.flags & ~NEXUS_SEG_K_ONLY) return NEXUS_EINVAL;
+    if (s.src_kind == NEXUS_SRC_BLOCK) {
+      if (s.src_index < 0 || s.src_index >= n_blocks) return NEXUS_ERANGE;
+      const nexus_status st = check_block(c, blocks[s.src_index]);
+      if (st != NEXUS_OK) return st;
+      if (s.src_start + static_cast<int64_t>(s.n_tokens) > blocks[s.src_index].n_tokens)
+        return NEXUS_ERANGE;
+    } else if (s.src_kind == NEXUS_SRC_CACHE) {
+      if (s.src_index < 0 || s.src_index >= n_rows) return NEXUS_ERANGE;
+      if (s.src_start + static_cast<int64_t>(s.n_tokens) > cap) return NEXUS_ERANGE;
+    } else {
+      return NEXUS_EINVAL;
+    }
+  }
+  if (!h_pt) return NEXUS_OK;
+
+  thread_local SlotMarks marks;
+  marks.ensure(c->n_pages * kPageSize);
+  nexus_status result = NEXUS_OK;
+  auto slot_of = [&](int32_t row, int32_t pos, int64_t* slot) -> bool {
+    const int32_t pg = h_pt[static_cast<int64_t>(row) * max_pages + pos / kPageSize];
+    if (pg < 0 || pg >= c->n_pages) return false;
+    *slot = static_cast<int64_t>(pg) * kPageSize + pos % kPageSize;
+    return true;
+  };
+  for (int32_t i = 0; i < n_segs && result == NEXUS_OK; ++i) {
+    const nexus_splice_segment& s = segs[i];
+    for (int32_t r = 0; r < s.n_tokens; ++r) {
+      int64_t slot;
+      if (!slot_of(s.dst_row, s.dst_start + r, &slot)) { result = NEXUS_ERANGE; break; }
+      if (marks.owner[slot] != -1) { result = NEXUS_EOVERLAP; break; }
+      marks.owner[slot] = i;
+      marks.touched.push_back(slot);
+    }
+  }
+  for (int32_t i = 0; i < n_segs && result == NEXUS_OK; ++i) {
+    const nexus_splice_segment& s = segs[i];
+    if (s.src_kind != NEXUS_SRC_CACHE) continue;
+    const bool in_place = (s.flags & NEXUS_SEG_K_ONLY) && s.src_index == s.dst_row &&
+                          s.src_start == s.dst_start;
+    for (int32_t r = 0; r < s.n_tokens; ++r) {
+      int64_t slot;
+      if (!slot_of(s.src_index, s.src_start + r, &slot)) { result = NEXUS_ERANGE; break; }
+      const int32_t o = marks.owner[slot];
+      if (o != -1 && !(o == i && in_place)) { result = NEXUS_EOVERLAP; break; }
+    }
+  }
+  marks.reset();
+  return result;
+}
+
+nexus_status launch_segments(const nexus_kv_cache* c, const int32_t* d_pt, int32_t max_pages,
+                             const nexus_block* blocks, const nexus_splice_segment* segs,
+                             int32_t n_segs, int32_t lb, int32_t le, int32_t out_mode,
+                             float* out_f32, int32_t out_pos_begin, cudaStream_t stream) {
+  std::unique_ptr<SpliceLaunch> p(new SpliceLaunch());
+  std::memset(p.get(), 0, sizeof(SpliceLaunch));
+  p->k_pool = static_cast<uint16_t*>(c->k_pool);
+  p->v_pool = static_cast<uint16_t*>(c->v_pool);
+  p->page_tables = d_pt;
+  p->out_f32 = out_f32;
+  p->n_pages = c->n_pages;
+  p->n_kv_heads = c->n_kv_heads;
+  p->max_pages = max_pages;
+  p->layer_begin = lb;
+  p->n_layers_call = le - lb;
+  p->v_transposed = c->v_transposed;
+  p->rope_gptj = c->rope_type == NEXUS_ROPE_GPTJ;
+  p->out_mode = out_mode;
+  p->out_pos_begin = out_pos_begin;
+  fill_inv_freq_over_pi(c, p->inv_freq_over_pi);
+  int32_t i = 0;
+  while (i < n_segs) {
+    int32_t ns = 0, pieces = 0;
+    for (; i < n_segs && ns < kMaxSegmentsPerLaunch; ++i) {
+      const nexus_splice_segment& s = segs[i];
+      const int32_t np = pieces_of(s.dst_start, s.n_tokens);
+      if (np == 0) continue;
+      DevSegment& d = p->seg[ns++];
+      if (s.src_kind == NEXUS_SRC_BLOCK) {
+        const nexus_block& b = blocks[s.src_index];
+        d.src_k = static_cast<const uint16_t*>(b.k);
+        d.src_v = static_cast<const uint16_t*>(b.v);
+        d.src_layer_stride = static_cast<int64_t>(b.n_tokens) * c->n_kv_heads * kHeadDim;
+        d.src_row = -1;
+      } else {
+        d.src_k = nullptr;
+        d.src_v = nullptr;
+        d.src_layer_stride = 0;
+        d.src_row = s.src_index;
+      }
+      d.src_start = s.src_start;
+      d.dst_row = s.dst_row;
+      d.dst_start = s.dst_start;
+      d.n_tokens = s.n_tokens;
+      d.delta = s.delta;
+      d.flags = s.flags;
+      d.piece_begin = pieces;
+      pieces += np;
+    }
+    if (ns == 0) continue;
+    p->n_segments = ns;
+    p->n_pieces = pieces;
+    if (launch_splice(*p, stream) != cudaSuccess) return NEXUS_ECUDA;
+  }
+  return NEXUS_OK;
+}
+
+// ------------------------------------------------------------- attention
+PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* f = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &f, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(f);
+    else
+      cudaGetLastError();
+  });
+  return fn;
+}
+
+bool encode_4d(CUtensorMap* m, const void* base, const uint64_t dims[4], const uint64_t strides[3],
+               const uint32_t box[4], CUtensorMapSwizzle swz) {
+  auto enc = tensor_map_encoder();
+  if (!enc) return false;
+  const cuuint32_t elem[4] = {1, 1, 1, 1};
+  const CUresult r =
+      enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(base),
+          reinterpret_cast<const cuuint64_t*>(dims), reinterpret_cast<const cuuint64_t*>(strides),
+          reinterpret_cast<const cuuint32_t*>(box), elem, CU_TENSOR_MAP_INTERLEAVE_NONE, swz,
+          CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
+struct AttnPlan {
+  int32_t total_tiles = 0;
+  int32_t n_tok = 0;
+  int32_t splits = 1;
+  int32_t kt_max = 0;
+};
+
+nexus_status plan_attention(int32_t n_seqs, const int32_t* kv_len, const int32_t* q_len,
+                            int32_t n_q_heads, int32_t n_kv_heads, int32_t n_layers_call,
+                            int32_t split_kv, AttnPlan* out) {
+  if (n_seqs < 1 || n_seqs > kMaxSeqs || !kv_len || !q_len) return NEXUS_EINVAL;
+  if (n_kv_heads < 1 || n_q_heads < n_kv_heads || n_q_heads % n_kv_heads != 0) return NEXUS_EINVAL;
+  const int32_t group = n_q_heads / n_kv_heads;
+  if (group > 128) return NEXUS_EINVAL;
+  const int32_t tile_tokens = 128 / group;
+  AttnPlan pl;
+  int64_t tok = 0, tiles = 0;
+  for (int32_t s = 0; s < n_seqs; ++s) {
+    if (q_len[s] < 0 || kv_len[s] < q_len[s]) return NEXUS_EINVAL;
+    tok += q_len[s];
+    tiles += (q_len[s] + tile_tokens - 1) / tile_tokens;
+    if (q_len[s] > 0) pl.kt_max = std::max(pl.kt_max, (kv_len[s] + 127) / 128);
+  }
+  if (tok > 0x7FFFFFFF || tiles > 0x7FFFFFFF) return NEXUS_ERANGE;
+  pl.n_tok = static_cast<int32_t>(tok);
+  pl.total_tiles = static_cast<int32_t>(tiles);
+  if (split_kv < 0) return NEXUS_EINVAL;
+  if (split_kv == 0) {
+    // Balance waves of one-CTA-per-SM work against the per-split merge.
+    const int64_t ctas = tiles * n_kv_heads * std::max(1, n_layers_call);
+    const int sms = num_sms();
+    int best = 1;
+    double best_cost = 1e300;
+    if (ctas > 0 && pl.kt_max > 0) {
+      for (int s = 1; s <= std::min<int>(kMaxSplits, pl.kt_max); ++s) {
+        const double waves = std::ceil(static_cast<double>(ctas) * s / sms);
+        const double cost = waves * std::ceil(static_cast<double>(pl.kt_max) / s) + (s > 1 ? 2.0 : 0.0);
+        if (cost < best_cost - 1e-9) { best_cost = cost; best = s; }
+      }
+    }
+    pl.splits = best;
+  } else {
+    pl.splits = std::min(split_kv, kMaxSplits);
+  }
+  *out = pl;
+  return NEXUS_OK;
+}
+
+size_t workspace_bytes_for(const AttnPlan& pl, int32_t n_q_heads, int32_t n_layers_call) {
+  if (pl.splits <= 1) return 0;
+  const size_t rows = static_cast<size_t>(pl.n_tok) * n_q_heads * n_layers_call;
+  return static_cast<size_t>(pl.splits) * rows * (kHeadDim * sizeof(float) + sizeof(float));
+}
+
+nexus_status attention_impl(const nexus_kv_cache* c, const int32_t* d_pt, int32_t n_rows,
+                            int32_t max_pages, int32_t n_seqs, const int32_t* h_rows,
+                            const int32_t* kv_len, const int32_t* q_len, const void* q, void* out,
+                            float* lse, int32_t n_q_heads, int32_t lb, int32_t le,
+                            int32_t split_kv, void* ws, size_t ws_bytes, cudaStream_t stream) {
+  nexus_status st = check_cache(c);
+  if (st != NEXUS_OK) return st;
+  if ((st = check_layers(c, lb, le)) != NEXUS_OK) return st;
+  if (!d_pt || n_rows < 1 || max_pages < 1 || !q || !out) return NEXUS_EINVAL;
+  if (!aligned16(q) || !aligned16(out) || (lse && (reinterpret_cast<uintptr_t>(lse) & 3u)))
+    return NEXUS_ELAYOUT;
+  AttnPlan pl;
+  if ((st = plan_attention(n_seqs, kv_len, q_len, n_q_heads, c->n_kv_heads, le - lb, split_kv,
+                           &pl)) != NEXUS_OK)
+    return st;
+  const int64_t cap = static_cast<int64_t>(max_pages) * kPageSize;
+  for (int32_t s = 0; s < n_seqs; ++s) {
+    const int32_t row = h_rows ? h_rows[s] : s;
+    if (row < 0 || row >= n_rows) return NEXUS_ERANGE;
+    if (kv_len[s] > cap) return NEXUS_ERANGE;
+  }
+  if (pl.n_tok == 0 || le == lb) return NEXUS_OK;
+  const size_t need = workspace_bytes_for(pl, n_q_heads, le - lb);
+  if (need > 0 && (!ws || ws_bytes < need || !aligned16(ws))) return NEXUS_ENOMEM;
+
+  std::unique_ptr<AttnLaunch> p(new AttnLaunch());
+  std::memset(p.get(), 0, sizeof(AttnLaunch));
+  const int32_t group = n_q_heads / c->n_kv_heads;
+  p->page_tables = d_pt;
+  p->out = static_cast<uint16_t*>(out);
+  p->lse = lse;
+  p->max_pages = max_pages;
+  p->n_q_heads = n_q_heads;
+  p->n_kv_heads = c->n_kv_heads;
+  p->group = group;
+  p->tile_tokens = 128 / group;
+  p->n_tok = pl.n_tok;
+  p->n_pages = static_cast<int32_t>(c->n_pages);
+  p->layer_begin = lb;
+  p->n_layers_call = le - lb;
+  p->n_seqs = n_seqs;
+  p->splits = pl.splits;
+  p->v_transposed = c->v_transposed;
+  p->total_tiles = pl.total_tiles;
+  p->scale_log2 = static_cast<float>(1.4426950408889634 / std::sqrt(static_cast<double>(kHeadDim)));
+  if (pl.splits > 1) {
+    const size_t rows = static_cast<size_t>(pl.n_tok) * n_q_heads * (le - lb);
+    p->part_o = static_cast<float*>(ws);
+    p->part_lse = static_cast<float*>(ws) + static_cast<size_t>(pl.splits) * rows * kHeadDim;
+  }
+  int32_t tiles = 0, off = 0;
+  for (int32_t s = 0; s < n_seqs; ++s) {
+    p->tile_prefix[s] = tiles;
+    p->seq[s].kv_len = kv_len[s];
+    p->seq[s].q_len = q_len[s];
+    p->seq[s].q_off = off;
+    p->seq[s].pt_row = h_rows ? h_rows[s] : s;
+    tiles += (q_len[s] + p->tile_tokens - 1) / p->tile_tokens;
+    off += q_len[s];
+  }
+  p->tile_prefix[n_seqs] = tiles;
+
+  AttnMaps maps;
+  const uint64_t tok_stride = static_cast<uint64_t>(n_q_heads) * kHeadDim * 2;
+  {
+    const uint64_t dims[4] = {kHeadDim, static_cast<uint64_t>(n_q_heads),
+                              static_cast<uint64_t>(pl.n_tok), static_cast<uint64_t>(le - lb)};
+    const uint64_t strides[3] = {kHeadDim * 2, tok_stride, tok_stride * pl.n_tok};
+    const uint32_t box[4] = {64, static_cast<uint32_t>(group), static_cast<uint32_t>(p->tile_tokens), 1};
+    if (!encode_4d(&maps.q, q, dims, strides, box, CU_TENSOR_MAP_SWIZZLE_128B)) return NEXUS_ECUDA;
+  }
+  const uint64_t head_bytes = kPageSize * kHeadDim * 2;   // 4 KiB per (page, head)
+  const uint64_t gpages = static_cast<uint64_t>(c->n_pages) * c->n_layers;
+  {
+    const uint64_t dims[4] = {kHeadDim, kPageSize, static_cast<uint64_t>(c->n_kv_heads), gpages};
+    const uint64_t strides[3] = {kHeadDim * 2, head_bytes, head_bytes * c->n_kv_heads};
+    const uint32_t box[4] = {64, kPageSize, 1, 1};
+    if (!encode_4d(&maps.k, c->k_pool, dims, strides, box, CU_TENSOR_MAP_SWIZZLE_128B))
+      return NEXUS_ECUDA;
+    if (!c->v_transposed) {
+      if (!encode_4d(&maps.v, c->v_pool, dims, strides, box, CU_TENSOR_MAP_SWIZZLE_128B))
+        return NEXUS_ECUDA;
+    }
+  }
+  if (c->v_transposed) {
+    const uint64_t dims[4] = {kPageSize, kHeadDim, static_cast<uint64_t>(c->n_kv_heads), gpages};
+    const uint64_t strides[3] = {kPageSize * 2, head_bytes, head_bytes * c->n_kv_heads};
+    const uint32_t box[4] = {kPageSize, kHeadDim, 1, 1};
+    if (!encode_4d(&maps.v, c->v_pool, dims, strides, box, CU_TENSOR_MAP_SWIZZLE_32B))
+      return NEXUS_ECUDA;
+  }
+  if (launch_attention(*p, maps, stream) != cudaSuccess) return NEXUS_ECUDA;
+  if (pl.splits > 1 && launch_attn_combine(*p, stream) != cudaSuccess) return NEXUS_ECUDA;
+  return NEXUS_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+nexus_status nexus_device_status(nexus_stream stream) {
+  unsigned int flag = 0;
+  if (attention_take_timeout(&flag, static_cast<cudaStream_t>(stream)) != cudaSuccess) {
+    cudaGetLastError();
+    return NEXUS_ECUDA;
+  }
+  return flag ? NEXUS_ETIMEOUT : NEXUS_OK;
+}
+
+nexus_status nexus_splice_kv(const nexus_kv_cache* cache, const int32_t* d_page_tables,
+                             const int32_t* h_page_tables, int32_t n_rows, int32_t max_pages,
+                             const nexus_block* blocks, int32_t n_blocks,
+                             const nexus_splice_segment* segments, int32_t n_segments,
+                             int32_t layer_begin, int32_t layer_end, nexus_stream stream) {
+  nexus_status st = check_cache(cache);
+  if (st != NEXUS_OK) return st;
+  if ((st = check_layers(cache, layer_begin, layer_end)) != NEXUS_OK) return st;
+  if (n_segments < 0 || n_segments > 4096 || n_blocks < 0 || (n_segments > 0 && !segments) ||
+      (n_blocks > 0 && !blocks) || !d_page_tables || n_rows < 1 || max_pages < 1)
+    return NEXUS_EINVAL;
+  if ((st = validate_segments(cache, h_page_tables, n_rows, max_pages, blocks, n_blocks, segments,
+                              n_segments)) != NEXUS_OK)
+    return st;
+  if (layer_end == layer_begin || n_segments == 0) return NEXUS_OK;
+  return launch_segments(cache, d_page_tables, max_pages, blocks, segments, n_segments,
+                         layer_begin, layer_end, kOutPool, nullptr, 0,
+                         static_cast<cudaStream_t>(stream));
+}
+
+nexus_status nexus_rope_rerotate(const nexus_kv_cache* cache, const int32_t* d_page_tables,
+                                 const int32_t* h_page_tables, int32_t n_rows, int32_t max_pages,
+                                 int32_t row, int32_t pos_begin, int32_t n_tokens, int32_t delta,
+                                 int32_t layer_begin, int32_t layer_end, nexus_stream stream) {
+  nexus_status st = check_cache(cache);
+  if (st != NEXUS_OK) return st;
+  if ((st = check_layers(cache, layer_begin, layer_end)) != NEXUS_OK) return st;
+  if (!d_page_tables || n_rows < 1 || max_pages < 1) return NEXUS_EINVAL;
+  nexus_splice_segment s{NEXUS_SRC_CACHE, row, pos_begin, row, pos_begin, n_tokens, delta,
+                         NEXUS_SEG_K_ONLY};
+  if ((st = validate_segments(cache, h_page_tables, n_rows, max_pages, nullptr, 0, &s, 1)) !=
+      NEXUS_OK)
+    return st;
+  if (layer_end == layer_begin || n_tokens == 0 || delta == 0) return NEXUS_OK;
+  return launch_segments(cache, d_page_tables, max_pages, nullptr, &s, 1, layer_begin, layer_end,
+                         kOutPool, nullptr, 0, static_cast<cudaStream_t>(stream));
+}
+
+nexus_status nexus_rope_rerotate_f32(const nexus_kv_cache* cache, const int32_t* d_page_tables,
+                                     const int32_t* h_page_tables, int32_t n_rows,
+                                     int32_t max_pages, int32_t row, int32_t pos_begin,
+                                     int32_t n_tokens, int32_t delta, int32_t layer_begin,
+                                     int32_t layer_end, float* out_f32, nexus_stream stream) {
+  nexus_status st = check_cache(cache);
+  if (st != NEXUS_OK) return st;
+  if ((st = check_layers(cache, layer_begin, layer_end)) != NEXUS_OK) return st;
+  if (!d_page_tables || n_rows < 1 || max_pages < 1 || !out_f32) return NEXUS_EINVAL;
+  if (!aligned16(out_f32)) return NEXUS_ELAYOUT;
+  nexus_splice_segment s{NEXUS_SRC_CACHE, row, pos_begin, row, pos_begin, n_tokens, delta,
+                         NEXUS_SEG_K_ONLY};
+  if ((st = validate_segments(cache, h_page_tables, n_rows, max_pages, nullptr, 0, &s, 1)) !=
+      NEXUS_OK)
+    return st;
+  if (layer_end == layer_begin || n_tokens == 0) return NEXUS_OK;
+  return launch_segments(cache, d_page_tables, max_pages, nullptr, &s, 1, layer_begin, layer_end,
+                         kOutF32, out_f32, pos_begin, static_cast<cudaStream_t>(stream));
+}
+
+nexus_status nexus_copy_pages(const nexus_kv_cache* cache, const int32_t* h_src_pages,
+                              const int32_t* h_dst_pages, int32_t n, int32_t layer_begin,
+                              int32_t layer_end, nexus_stream stream) {
+  nexus_status st = check_cache(cache);
+  if (st != NEXUS_OK) return st;
+  if ((st = check_layers(cache, layer_begin, layer_end)) != NEXUS_OK) return st;
+  if (n < 0 || n > kMaxPageCopies || (n > 0 && (!h_src_pages || !h_dst_pages))) return NEXUS_EINVAL;
+  std::vector<int32_t> dst(h_dst_pages, h_dst_pages + n);
+  for (int32_t i = 0; i < n; ++i)
+    if (h_src_pages[i] < 0 || h_src_pages[i] >= cache->n_pages || h_dst_pages[i] < 0 ||
+        h_dst_pages[i] >= cache->n_pages)
+      return NEXUS_ERANGE;
+  std::sort(dst.begin(), dst.end());
+  if (std::adjacent_find(dst.begin(), dst.end()) != dst.end()) return NEXUS_EOVERLAP;
+  for (int32_t i = 0; i < n; ++i)
+    if (std::binary_search(dst.begin(), dst.end(), h_src_pages[i])) return NEXUS_EOVERLAP;
+  if (n == 0 || layer_end == layer_begin) return NEXUS_OK;
+  std::unique_ptr<PageCopyLaunch> p(new PageCopyLaunch());
+  p->k_pool = static_cast<uint16_t*>(cache->k_pool);
+  p->v_pool = static_cast<uint16_t*>(cache->v_pool);
+  p->n_pages = cache->n_pages;
+  p->n_kv_heads = cache->n_kv_heads;
+  p->layer_begin = layer_begin;
+  p->n_layers_call = layer_end - layer_begin;
+  p->n = n;
+  std::memcpy(p->src, h_src_pages, sizeof(int32_t) * n);
+  std::memcpy(p->dst, h_dst_pages, sizeof(int32_t) * n);
+  return launch_page_copy(*p, static_cast<cudaStream_t>(stream)) == cudaSuccess ? NEXUS_OK
+                                                                                 : NEXUS_ECUDA;
+}
+
+nexus_status nexus_suffix_attention(const nexus_kv_cache* cache, const int32_t* d_page_tables,
+                                    int32_t n_rows, int32_t max_pages, int32_t n_seqs,
+                                    const int32_t* h_rows, const int32_t* h_kv_len,
+                                    const int32_t* h_q_len, const void* q, void* out, float* lse,
+                                    int32_t n_q_heads, int32_t layer_begin, int32_t layer_end,
+                                    int32_t split_kv, void* workspace, size_t workspace_bytes,
+                                    nexus_stream stream) {
+  return attention_impl(cache, d_page_tables, n_rows, max_pages, n_seqs, h_rows, h_kv_len, h_q_len,
+                        q, out, lse, n_q_heads, layer_begin, layer_end, split_kv, workspace,
+                        workspace_bytes, static_cast<cudaStream_t>(stream));
+}
+
+nexus_status nexus_reprefill(const nexus_kv_cache* cache, const int32_t* d_page_tables,
+                             int32_t n_rows, int32_t max_pages, int32_t n_seqs,
+                             const int32_t* h_rows, const int32_t* h_kv_len, const void* q,
+                             void* out, float* lse, int32_t n_q_heads, int32_t layer_begin,
+                             int32_t layer_end, int32_t split_kv, void* workspace,
+                             size_t workspace_bytes, nexus_stream stream) {
+  return attention_impl(cache, d_page_tables, n_rows, max_pages, n_seqs, h_rows, h_kv_len, h_kv_len,
+                        q, out, lse, n_q_heads, layer_begin, layer_end, split_kv, workspace,
+                        workspace_bytes, static_cast<cudaStream_t>(stream));
+}
+
+size_t nexus_attention_workspace_size(int32_t n_seqs, const int32_t* h_kv_len,
+                                      const int32_t* h_q_len, int32_t n_q_heads,
+                                      int32_t n_kv_heads, int32_t n_layers_call, int32_t split_kv,
+                                      int32_t* splits_out) {
+  AttnPlan pl;
+  if (plan_attention(n_seqs, h_kv_len, h_q_len, n_q_heads, n_kv_heads, n_layers_call, split_kv,
+                     &pl) != NEXUS_OK) {
+    if (splits_out) *splits_out = 0;
+    return 0;
+  }
+  if (splits_out) *splits_out = pl.splits;
+  return workspace_bytes_for(pl, n_q_heads, n_layers_call);
+}
+
+}  // extern "C"

@@ -1,0 +1,359 @@
+"""Thin ctypes binding of ``libnexus.so`` (see ``include/nexus.h``).
+
+Argument marshalling only: every step of the path runs in the library's CUDA
+kernels or its C++ host runtime. Device buffers may be given as torch tensors
+(their ``data_ptr()`` is passed) or as raw integer addresses; torch supplies
+device memory and streams, nothing else. Importing this module does not load
+the library; the first call does, and it raises ``NexusLibraryMissing`` if the
+library has not been built (there is no fallback of any kind).
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from ctypes import POINTER, c_double, c_int32, c_int64, c_size_t, c_void_p
+from fractions import Fraction
+from typing import Optional, Sequence
+
+import numpy as np
+
+LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "libnexus.so")
+
+OK, EINVAL, ERANGE, EROPE_MISMATCH, ELAYOUT, ENOMEM, EDECLINED, ECUDA, ETIMEOUT, EOVERLAP = range(10)
+ROPE_NEOX, ROPE_GPTJ = 0, 1
+SRC_BLOCK, SRC_CACHE = 0, 1
+SEG_K_ONLY = 1
+
+
+class NexusLibraryMissing(RuntimeError):
+    pass
+
+
+class NexusError(RuntimeError):
+    def __init__(self, fn: str, code: int):
+        self.code = int(code)
+        super().__init__(f"{fn}: {status_string(code)} (status {code})")
+
+
+class KvCache(ctypes.Structure):
+    _fields_ = [
+        ("k_pool", c_void_p), ("v_pool", c_void_p), ("n_pages", c_int64),
+        ("n_layers", c_int32), ("n_kv_heads", c_int32), ("head_dim", c_int32),
+        ("page_size", c_int32), ("v_transposed", c_int32), ("rope_type", c_int32),
+        ("rope_theta", c_double), ("rope_freq_scale", c_double),
+    ]
+
+
+class Block(ctypes.Structure):
+    _fields_ = [
+        ("k", c_void_p), ("v", c_void_p), ("n_tokens", c_int32), ("base_pos", c_int32),
+        ("n_layers", c_int32), ("n_kv_heads", c_int32), ("head_dim", c_int32),
+        ("rope_type", c_int32), ("rope_theta", c_double), ("rope_freq_scale", c_double),
+    ]
+
+
+class Segment(ctypes.Structure):
+    _fields_ = [
+        ("src_kind", c_int32), ("src_index", c_int32), ("src_start", c_int32),
+        ("dst_row", c_int32), ("dst_start", c_int32), ("n_tokens", c_int32),
+        ("delta", c_int32), ("flags", c_int32),
+    ]
+
+
+class Policy(ctypes.Structure):
+    _fields_ = [("splice_threshold", c_int32), ("r_base_pct", c_int32), ("full_mult", c_int32)]
+
+
+class Insert(ctypes.Structure):
+    _fields_ = [("depth", c_int32), ("block_index", c_int32)]
+
+
+DEFAULT_POLICY = (256, 5, 4)   # P = M = 256, R_base = 5 %, K = 4 (Sec. III-B / III-C)
+
+_i32p = POINTER(c_int32)
+_SIGS = {
+    "nexus_status_string": (ctypes.c_char_p, [c_int32]),
+    "nexus_version": (c_int32, []),
+    "nexus_device_status": (c_int32, [c_void_p]),
+    "nexus_recompute_pct": (c_int32, [c_int32, POINTER(Policy), POINTER(c_int64), POINTER(c_int64)]),
+    "nexus_redecode_len": (c_int32, [c_int32, c_int32, POINTER(Policy)]),
+    "nexus_suffix_len": (c_int32, [c_int32, c_int32]),
+    "nexus_check_splice": (c_int32, [c_int32, c_int32, c_int32, POINTER(Policy)]),
+    "nexus_page_pool_create": (c_int32, [c_int64, _i32p, POINTER(c_void_p)]),
+    "nexus_page_pool_destroy": (None, [c_void_p]),
+    "nexus_page_pool_alloc": (c_int32, [c_void_p, c_int32, _i32p]),
+    "nexus_page_pool_free": (c_int32, [c_void_p, c_int32, _i32p]),
+    "nexus_page_pool_available": (c_int64, [c_void_p]),
+    "nexus_plan_splice": (c_int32, [c_void_p, _i32p, c_int32, c_int32, POINTER(Block), c_int32,
+                                    POINTER(Insert), c_int32, c_int32, c_int32, _i32p,
+                                    POINTER(Segment), c_int32, _i32p, _i32p, _i32p]),
+    "nexus_splice_kv": (c_int32, [POINTER(KvCache), c_void_p, _i32p, c_int32, c_int32,
+                                  POINTER(Block), c_int32, POINTER(Segment), c_int32,
+                                  c_int32, c_int32, c_void_p]),
+    "nexus_rope_rerotate": (c_int32, [POINTER(KvCache), c_void_p, _i32p, c_int32, c_int32, c_int32,
+                                      c_int32, c_int32, c_int32, c_int32, c_int32, c_void_p]),
+    "nexus_rope_rerotate_f32": (c_int32, [POINTER(KvCache), c_void_p, _i32p, c_int32, c_int32,
+                                          c_int32, c_int32, c_int32, c_int32, c_int32, c_int32,
+                                          c_void_p, c_void_p]),
+    "nexus_copy_pages": (c_int32, [POINTER(KvCache), _i32p, _i32p, c_int32, c_int32, c_int32,
+                                   c_void_p]),
+    "nexus_suffix_attention": (c_int32, [POINTER(KvCache), c_void_p, c_int32, c_int32, c_int32,
+                                         _i32p, _i32p, _i32p, c_void_p, c_void_p, c_void_p,
+                                         c_int32, c_int32, c_int32, c_int32, c_void_p, c_size_t,
+                                         c_void_p]),
+    "nexus_reprefill": (c_int32, [POINTER(KvCache), c_void_p, c_int32, c_int32, c_int32, _i32p,
+                                  _i32p, c_void_p, c_void_p, c_void_p, c_int32, c_int32, c_int32,
+                                  c_int32, c_void_p, c_size_t, c_void_p]),
+    "nexus_attention_workspace_size": (c_size_t, [c_int32, _i32p, _i32p, c_int32, c_int32,
+                                                  c_int32, c_int32, _i32p]),
+}
+EXPORTED = tuple(_SIGS)
+
+_lib = None
+
+
+def lib():
+    """The loaded library; raises NexusLibraryMissing if it was never built."""
+    global _lib
+    if _lib is None:
+        if not os.path.exists(LIB_PATH):
+            raise NexusLibraryMissing(
+                f"{LIB_PATH} is missing: build it with __graft_entry__.build() (no fallback exists)")
+        L = ctypes.CDLL(LIB_PATH)
+        for name, (res, args) in _SIGS.items():
+            f = getattr(L, name)
+            f.restype = res
+            f.argtypes = args
+        _lib = L
+    return _lib
+
+
+def status_string(code: int) -> str:
+    return lib().nexus_status_string(int(code)).decode()
+
+
+def _check(fn: str, code: int):
+    if code != OK:
+        raise NexusError(fn, code)
+
+
+def _ptr(x) -> Optional[int]:
+    if x is None:
+        return None
+    if isinstance(x, int):
+        return x
+    return int(x.data_ptr())
+
+
+def _i32(a) -> Optional[ctypes.Array]:
+    """A host int32 array as a ctypes buffer (kept alive by the caller's scope)."""
+    if a is None:
+        return None
+    arr = np.ascontiguousarray(np.asarray(a, dtype=np.int32))
+    return arr.ctypes.data_as(_i32p), arr
+
+
+def _stream(stream) -> Optional[int]:
+    if stream is None:
+        import torch
+        return int(torch.cuda.current_stream().cuda_stream)
+    if isinstance(stream, int):
+        return stream
+    return int(stream.cuda_stream)
+
+
+def _policy(policy) -> Policy:
+    p = policy if policy is not None else DEFAULT_POLICY
+    return Policy(int(p[0]), int(p[1]), int(p[2]))
+
+
+# ---------------------------------------------------------------- policy
+def recompute_pct(n_past: int, policy=None) -> Fraction:
+    num, den = c_int64(), c_int64()
+    pol = _policy(policy)
+    _check("nexus_recompute_pct", lib().nexus_recompute_pct(int(n_past), ctypes.byref(pol),
+                                                            ctypes.byref(num), ctypes.byref(den)))
+    return Fraction(num.value, den.value)
+
+
+def redecode_len(S: int, n_past: int, policy=None) -> int:
+    pol = _policy(policy)
+    r = lib().nexus_redecode_len(int(S), int(n_past), ctypes.byref(pol))
+    if r < 0:
+        raise NexusError("nexus_redecode_len", EINVAL)
+    return int(r)
+
+
+def suffix_len(S: int, pct: int) -> int:
+    r = lib().nexus_suffix_len(int(S), int(pct))
+    if r < 0:
+        raise NexusError("nexus_suffix_len", EINVAL)
+    return int(r)
+
+
+def check_splice(n_past: int, S: int, n_redecode: int, policy=None) -> int:
+    pol = _policy(policy)
+    return int(lib().nexus_check_splice(int(n_past), int(S), int(n_redecode), ctypes.byref(pol)))
+
+
+# ------------------------------------------------------------- page pool
+class PagePool:
+    def __init__(self, n_pages: int, order: Optional[Sequence[int]] = None):
+        h = c_void_p()
+        buf = _i32(order)
+        _check("nexus_page_pool_create",
+               lib().nexus_page_pool_create(int(n_pages), buf[0] if buf else None, ctypes.byref(h)))
+        self._h = h
+        self.n_pages = int(n_pages)
+
+    @property
+    def handle(self):
+        return self._h
+
+    def alloc(self, n: int) -> np.ndarray:
+        out = np.zeros(int(n), dtype=np.int32)
+        _check("nexus_page_pool_alloc",
+               lib().nexus_page_pool_alloc(self._h, int(n), out.ctypes.data_as(_i32p)))
+        return out
+
+    def free(self, pages) -> None:
+        buf = _i32(pages)
+        _check("nexus_page_pool_free", lib().nexus_page_pool_free(self._h, len(buf[1]), buf[0]))
+
+    def available(self) -> int:
+        return int(lib().nexus_page_pool_available(self._h))
+
+    def close(self):
+        if self._h:
+            lib().nexus_page_pool_destroy(self._h)
+            self._h = c_void_p()
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+
+# -------------------------------------------------------------- structs
+def kv_cache(k_pool, v_pool, n_pages: int, n_layers: int, n_kv_heads: int = 8,
+             v_transposed: bool = False, rope_type: int = ROPE_NEOX, rope_theta: float = 1.0e6,
+             rope_freq_scale: float = 1.0) -> KvCache:
+    return KvCache(_ptr(k_pool), _ptr(v_pool), int(n_pages), int(n_layers), int(n_kv_heads), 128,
+                   16, int(bool(v_transposed)), int(rope_type), float(rope_theta),
+                   float(rope_freq_scale))
+
+
+def block(k, v, n_tokens: int, base_pos: int, n_layers: int, n_kv_heads: int = 8,
+          rope_type: int = ROPE_NEOX, rope_theta: float = 1.0e6,
+          rope_freq_scale: float = 1.0) -> Block:
+    return Block(_ptr(k), _ptr(v), int(n_tokens), int(base_pos), int(n_layers), int(n_kv_heads),
+                 128, int(rope_type), float(rope_theta), float(rope_freq_scale))
+
+
+def segments_array(segs) -> ctypes.Array:
+    arr = (Segment * max(1, len(segs)))()
+    for i, s in enumerate(segs):
+        arr[i] = s if isinstance(s, Segment) else Segment(*[int(x) for x in s])
+    return arr
+
+
+# --------------------------------------------------------------- planner
+def plan_splice(pool: PagePool, old_pt, n_past: int, max_pages: int, blocks: Sequence[Block],
+                inserts: Sequence[tuple], old_row: int, new_row: int, seg_capacity: int = 64):
+    """Returns (new_pt [max_pages] int32, list of Segment, freed pages)."""
+    barr = (Block * max(1, len(blocks)))(*blocks)
+    iarr = (Insert * max(1, len(inserts)))(*[Insert(int(d), int(b)) for d, b in inserts])
+    old = _i32(old_pt if old_pt is not None else np.zeros(max_pages, np.int32))
+    new_pt = np.zeros(int(max_pages), dtype=np.int32)
+    segs = (Segment * seg_capacity)()
+    nseg = c_int32()
+    freed = np.zeros(int(max_pages), dtype=np.int32)
+    nfreed = c_int32()
+    _check("nexus_plan_splice", lib().nexus_plan_splice(
+        pool.handle, old[0], int(n_past), int(max_pages), barr, len(blocks), iarr, len(inserts),
+        int(old_row), int(new_row), new_pt.ctypes.data_as(_i32p), segs, int(seg_capacity),
+        ctypes.byref(nseg), freed.ctypes.data_as(_i32p), ctypes.byref(nfreed)))
+    return new_pt, [segs[i] for i in range(nseg.value)], freed[: nfreed.value].copy()
+
+
+# ---------------------------------------------------------------- device
+def splice_kv(cache: KvCache, d_page_tables, h_page_tables, n_rows: int, max_pages: int,
+              blocks: Sequence[Block], segments, layer_begin: int, layer_end: int, stream=None):
+    barr = (Block * max(1, len(blocks)))(*blocks)
+    sarr = segments_array(segments)
+    hpt = _i32(h_page_tables)
+    _check("nexus_splice_kv", lib().nexus_splice_kv(
+        ctypes.byref(cache), _ptr(d_page_tables), hpt[0] if hpt else None, int(n_rows),
+        int(max_pages), barr, len(blocks), sarr, len(segments), int(layer_begin), int(layer_end),
+        _stream(stream)))
+
+
+def rope_rerotate(cache: KvCache, d_page_tables, h_page_tables, n_rows: int, max_pages: int,
+                  row: int, pos_begin: int, n_tokens: int, delta: int, layer_begin: int,
+                  layer_end: int, stream=None):
+    hpt = _i32(h_page_tables)
+    _check("nexus_rope_rerotate", lib().nexus_rope_rerotate(
+        ctypes.byref(cache), _ptr(d_page_tables), hpt[0] if hpt else None, int(n_rows),
+        int(max_pages), int(row), int(pos_begin), int(n_tokens), int(delta), int(layer_begin),
+        int(layer_end), _stream(stream)))
+
+
+def rope_rerotate_f32(cache: KvCache, d_page_tables, h_page_tables, n_rows: int, max_pages: int,
+                      row: int, pos_begin: int, n_tokens: int, delta: int, layer_begin: int,
+                      layer_end: int, out_f32, stream=None):
+    hpt = _i32(h_page_tables)
+    _check("nexus_rope_rerotate_f32", lib().nexus_rope_rerotate_f32(
+        ctypes.byref(cache), _ptr(d_page_tables), hpt[0] if hpt else None, int(n_rows),
+        int(max_pages), int(row), int(pos_begin), int(n_tokens), int(delta), int(layer_begin),
+        int(layer_end), _ptr(out_f32), _stream(stream)))
+
+
+def copy_pages(cache: KvCache, src_pages, dst_pages, layer_begin: int, layer_end: int, stream=None):
+    s = _i32(src_pages)
+    d = _i32(dst_pages)
+    _check("nexus_copy_pages", lib().nexus_copy_pages(
+        ctypes.byref(cache), s[0], d[0], len(s[1]), int(layer_begin), int(layer_end),
+        _stream(stream)))
+
+
+def attention_workspace_size(kv_len, q_len, n_q_heads: int, n_kv_heads: int, n_layers_call: int,
+                             split_kv: int = 0):
+    kv = _i32(kv_len)
+    ql = _i32(q_len)
+    splits = c_int32()
+    n = lib().nexus_attention_workspace_size(len(kv[1]), kv[0], ql[0], int(n_q_heads),
+                                             int(n_kv_heads), int(n_layers_call), int(split_kv),
+                                             ctypes.byref(splits))
+    return int(n), int(splits.value)
+
+
+def suffix_attention(cache: KvCache, d_page_tables, n_rows: int, max_pages: int, kv_len, q_len,
+                     q, out, lse=None, n_q_heads: int = 40, layer_begin: int = 0,
+                     layer_end: int = 1, rows=None, split_kv: int = 0, workspace=None,
+                     workspace_bytes: int = 0, stream=None):
+    kv = _i32(kv_len)
+    ql = _i32(q_len)
+    rw = _i32(rows)
+    _check("nexus_suffix_attention", lib().nexus_suffix_attention(
+        ctypes.byref(cache), _ptr(d_page_tables), int(n_rows), int(max_pages), len(kv[1]),
+        rw[0] if rw else None, kv[0], ql[0], _ptr(q), _ptr(out), _ptr(lse), int(n_q_heads),
+        int(layer_begin), int(layer_end), int(split_kv), _ptr(workspace), int(workspace_bytes),
+        _stream(stream)))
+
+
+def reprefill(cache: KvCache, d_page_tables, n_rows: int, max_pages: int, kv_len, q, out,
+              lse=None, n_q_heads: int = 40, layer_begin: int = 0, layer_end: int = 1, rows=None,
+              split_kv: int = 1, workspace=None, workspace_bytes: int = 0, stream=None):
+    kv = _i32(kv_len)
+    rw = _i32(rows)
+    _check("nexus_reprefill", lib().nexus_reprefill(
+        ctypes.byref(cache), _ptr(d_page_tables), int(n_rows), int(max_pages), len(kv[1]),
+        rw[0] if rw else None, kv[0], _ptr(q), _ptr(out), _ptr(lse), int(n_q_heads),
+        int(layer_begin), int(layer_end), int(split_kv), _ptr(workspace), int(workspace_bytes),
+        _stream(stream)))
+
+
+def device_status(stream=None) -> int:
+    """Synchronises the stream; OK, ETIMEOUT (a bounded device wait gave up) or ECUDA."""
+    return int(lib().nexus_device_status(_stream(stream)))

@@ -1,0 +1,209 @@
+"""Suffix-redecode / re-prefill attention on the GPU against the fp64 oracle
+(softmax(QK^T / sqrt(d)) V of Sec. III-A over the last R positions,
+Sec. III-C / Sec. V-A)."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from gpu_cases import (SplicedCase, assert_attn_close, f64, new_pools, write_rows)
+from paper_2608_20397_gb300 import nexus
+from paper_2608_20397_gb300.workloads import randn_bf16, workload
+
+pytestmark = pytest.mark.gpu
+DEV = torch.device("cuda:0") if torch.cuda.is_available() else None
+
+
+def _direct_case(kv_lens, q_lens, Hq=40, H=8, L=1, vt=False, seed=0, shuffle=True,
+                 garbage=True):
+    """Sequences written straight into a paged pool (no splice); slots past
+    kv_len hold NaN so any leak of them into the output shows."""
+    rng = np.random.default_rng(seed)
+    max_pages = max(-(-k // 16) for k in kv_lens) + 1
+    n_pages = sum(-(-k // 16) for k in kv_lens) + 8
+    kp, vp = new_pools(L, n_pages, H, vt, DEV, float("nan") if garbage else 0.0)
+    order = rng.permutation(n_pages) if shuffle else np.arange(n_pages)
+    h_pt = np.full((len(kv_lens), max_pages), -1, np.int32)
+    ks, vs, cur = [], [], 0
+    for i, T in enumerate(kv_lens):
+        npg = -(-T // 16)
+        h_pt[i, :npg] = order[cur:cur + npg]
+        cur += npg
+        k = randn_bf16((L, T, H, 128), seed * 100 + 2 * i, DEV)
+        v = randn_bf16((L, T, H, 128), seed * 100 + 2 * i + 1, DEV)
+        write_rows(kp, vp, h_pt[i], k, v, vt)
+        ks.append(k)
+        vs.append(v)
+    q = randn_bf16((L, sum(q_lens), Hq, 128), seed * 100 + 99, DEV)
+    cache = nexus.kv_cache(kp, vp, n_pages, L, H, vt)
+    return cache, torch.as_tensor(h_pt, device=DEV), max_pages, ks, vs, q
+
+
+def _run(cache, d_pt, max_pages, kv_lens, q_lens, q, Hq, L, split_kv=1, rows=None):
+    o = torch.full_like(q, float("nan"))
+    lse = torch.full(q.shape[:3], float("nan"), dtype=torch.float32, device=DEV)
+    nbytes, _ = nexus.attention_workspace_size(kv_lens, q_lens, Hq, cache.n_kv_heads, L, split_kv)
+    ws = torch.empty(max(nbytes, 16), dtype=torch.uint8, device=DEV)
+    nexus.suffix_attention(cache, d_pt, d_pt.shape[0], max_pages, kv_lens, q_lens, q, o, lse, Hq,
+                           0, L, rows=rows, split_kv=split_kv, workspace=ws, workspace_bytes=nbytes)
+    assert nexus.device_status() == nexus.OK
+    return o, lse
+
+
+def _check(ks, vs, q, o, lse, kv_lens, q_lens, group, layer=0, what=""):
+    off = 0
+    for i, (T, R) in enumerate(zip(kv_lens, q_lens)):
+        if R == 0:
+            continue
+        want_o, want_l = oracle.attention(f64(q[layer, off:off + R]), f64(ks[i][layer]),
+                                          f64(vs[i][layer]), oracle.suffix_positions(T, R), group)
+        assert_attn_close(f64(o[layer, off:off + R]), want_o, f64(lse[layer, off:off + R]), want_l,
+                          f"{what} seq {i} T={T} R={R}")
+        off += R
+
+
+@pytest.mark.parametrize("T,R", [(1, 1), (2, 2), (15, 15), (16, 16), (17, 17), (130, 1),
+                                 (640, 64), (300, 24), (301, 25), (302, 26), (1000, 127),
+                                 (1001, 128), (1003, 129), (257, 257)])
+def test_suffix_attention_shapes(T, R):
+    cache, d_pt, mp, ks, vs, q = _direct_case([T], [R], seed=T * 7 + R)
+    o, lse = _run(cache, d_pt, mp, [T], [R], q, 40, 1)
+    _check(ks, vs, q, o, lse, [T], [R], 5, what="shape")
+
+
+@pytest.mark.parametrize("Hq,H", [(8, 8), (16, 2), (32, 8), (12, 4)])
+def test_gqa_groupings(Hq, H):
+    cache, d_pt, mp, ks, vs, q = _direct_case([333], [200], Hq=Hq, H=H, seed=Hq + H)
+    o, lse = _run(cache, d_pt, mp, [333], [200], q, Hq, 1)
+    _check(ks, vs, q, o, lse, [333], [200], Hq // H, what=f"gqa {Hq}/{H}")
+
+
+def test_transposed_v_layout():
+    cache, d_pt, mp, ks, vs, q = _direct_case([777], [300], vt=True, seed=3)
+    o, lse = _run(cache, d_pt, mp, [777], [300], q, 40, 1)
+    _check(ks, vs, q, o, lse, [777], [300], 5, what="vT")
+
+
+def test_varlen_batch_multi_layer():
+    kv = [700, 33, 1500, 16, 900]
+    ql = [100, 33, 7, 0, 450]
+    cache, d_pt, mp, ks, vs, q = _direct_case(kv, ql, L=3, seed=5)
+    o, lse = _run(cache, d_pt, mp, kv, ql, q, 40, 3)
+    for layer in range(3):
+        _check(ks, vs, q, o, lse, kv, ql, 5, layer, what=f"varlen layer {layer}")
+
+
+@pytest.mark.parametrize("splits", [2, 5, 19, 32])
+def test_split_kv_matches_oracle(splits):
+    kv, ql = [5000], [64]
+    cache, d_pt, mp, ks, vs, q = _direct_case(kv, ql, seed=11)
+    o, lse = _run(cache, d_pt, mp, kv, ql, q, 40, 1, split_kv=splits)
+    _check(ks, vs, q, o, lse, kv, ql, 5, what=f"split {splits}")
+
+
+def test_split_kv_auto_varlen():
+    kv, ql = [3000, 200, 4100], [40, 1, 64]
+    cache, d_pt, mp, ks, vs, q = _direct_case(kv, ql, L=2, seed=12)
+    _, splits = nexus.attention_workspace_size(kv, ql, 40, 8, 2, 0)
+    assert splits > 1
+    o, lse = _run(cache, d_pt, mp, kv, ql, q, 40, 2, split_kv=0)
+    for layer in range(2):
+        _check(ks, vs, q, o, lse, kv, ql, 5, layer, what="auto split")
+
+
+def test_reprefill_equals_textbook_causal():
+    T = 600
+    cache, d_pt, mp, ks, vs, q = _direct_case([T], [T], seed=13)
+    o = torch.empty_like(q)
+    lse = torch.empty(q.shape[:3], dtype=torch.float32, device=DEV)
+    nexus.reprefill(cache, d_pt, 1, mp, [T], q, o, lse, 40, 0, 1)
+    assert nexus.device_status() == nexus.OK
+    _check(ks, vs, q, o, lse, [T], [T], 5, what="reprefill")
+
+
+def test_attention_repeat_runs_bit_stable():
+    cache, d_pt, mp, ks, vs, q = _direct_case([2000], [300], seed=14)
+    o1, l1 = _run(cache, d_pt, mp, [2000], [300], q, 40, 1)
+    o2, l2 = _run(cache, d_pt, mp, [2000], [300], q, 40, 1)
+    assert torch.equal(o1.view(torch.int16), o2.view(torch.int16))
+    assert torch.equal(l1, l2)
+
+
+# ------------------------------------------------------- end to end
+def _e2e_session(case, si, R, layers, Hq=40, split_kv=1, sample_rows=None, seed=0):
+    """Splice already done; attention of the last R positions over the spliced
+    cache on `layers`, checked against oracle splice + oracle attention."""
+    w = case.w
+    s = w.sessions[si]
+    T = w.spliced_len(s)
+    q = randn_bf16((len(layers), R, Hq, 128), 5000 + seed, DEV)
+    o = torch.empty_like(q)
+    lse = torch.empty(q.shape[:3], dtype=torch.float32, device=DEV)
+    nbytes, _ = nexus.attention_workspace_size([T], [R], Hq, w.n_kv_heads, 1, split_kv)
+    ws = torch.empty(max(nbytes, 16), dtype=torch.uint8, device=DEV)
+    for li, layer in enumerate(layers):
+        nexus.suffix_attention(case.cache, case.d_pt, case.n_rows, case.max_pages, [T], [R],
+                               q[li:li + 1], o[li:li + 1], lse[li:li + 1], Hq, layer, layer + 1,
+                               rows=[2 * si + 1], split_kv=split_kv, workspace=ws,
+                               workspace_bytes=nbytes)
+    assert nexus.device_status() == nexus.OK
+    for li, layer in enumerate(layers):
+        want_k, want_v = oracle.splice_sequence(f64(case.live_k[si][[layer]]),
+                                                f64(case.live_v[si][[layer]]),
+                                                case.inserts_f64(si, [layer]), w.rope_theta)
+        rows = np.arange(R) if sample_rows is None else sample_rows
+        pos = oracle.suffix_positions(T, R)[rows]
+        kmax = int(pos.max()) + 1
+        want_o, want_l = oracle.attention(f64(q[li, rows]), want_k[0, :kmax], want_v[0, :kmax],
+                                          pos, Hq // w.n_kv_heads)
+        assert_attn_close(f64(o[li, rows]), want_o, f64(lse[li, rows]), want_l,
+                          f"e2e layer {layer}")
+
+
+@pytest.mark.parametrize("name", ["c1", "c2"])
+def test_end_to_end_single_layer(name):
+    w = workload(name)
+    case = SplicedCase(w, DEV)
+    case.splice()
+    s = w.sessions[0]
+    R = nexus.suffix_len(s.suffix_span, s.suffix_pct)
+    assert R == oracle.redecode_len(s.suffix_span, 0, 256, s.suffix_pct, 4)
+    _e2e_session(case, 0, R, [0])
+
+
+@pytest.mark.parametrize("pct", [25, 50, 100])
+def test_end_to_end_c3_transposed_v(pct):
+    w = workload("c3")
+    case = SplicedCase(w, DEV)
+    case.splice()
+    R = nexus.suffix_len(2192, pct)
+    rows = np.random.default_rng(pct).choice(R, size=min(R, 96), replace=False)
+    _e2e_session(case, 0, R, [0, 47], sample_rows=np.sort(rows), seed=pct)
+
+
+def test_end_to_end_c5_split_kv_full_size():
+    w = workload("c5")
+    case = SplicedCase(w, DEV)
+    case.splice()
+    _e2e_session(case, 0, 64, [5, 40], split_kv=0, seed=7)
+
+
+def test_c5_reprefill_full_size_sampled_rows():
+    """Path B: causal self-attention of the 32768-token pre-splice context."""
+    w = workload("c5")
+    case = SplicedCase(w, DEV)
+    T = w.sessions[0].n_past
+    layer = 17
+    q = randn_bf16((1, T, 40, 128), 777, DEV)
+    o = torch.empty_like(q)
+    lse = torch.empty(q.shape[:3], dtype=torch.float32, device=DEV)
+    nexus.reprefill(case.cache, case.d_pt, case.n_rows, case.max_pages, [T], q, o, lse, 40,
+                    layer, layer + 1, rows=[0])
+    assert nexus.device_status() == nexus.OK
+    rng = np.random.default_rng(3)
+    rows = np.sort(np.concatenate([[0, 1, 24, 25, 127, 128, T - 1],
+                                   rng.choice(T, size=57, replace=False)]))
+    kmax = int(rows.max()) + 1
+    want_o, want_l = oracle.attention(f64(q[0, rows]), f64(case.live_k[0][layer, :kmax]),
+                                      f64(case.live_v[0][layer, :kmax]), rows, 5)
+    assert_attn_close(f64(o[0, rows]), want_o, f64(lse[0, rows]), want_l, "c5 reprefill")
