@@ -1,0 +1,521 @@
+"""Benchmark of the Nexus KV-cache splicing hot path on GB300.
+
+One step = one pass of the whole path over the deep-context workload "c5"
+(Qwen2.5-14B attention shape: 40 query / 8 KV heads, d = 128, 48 layers,
+bf16, 16-token pages):
+
+  1. splice: a 2048-token compiled block (anchor 0) inserted at depth 30000 of
+     a 32768-token live cache, every layer, K reanchored by delta = 30000 and
+     the 2768 displaced rows re-rotated by +2048 (one launch);
+  2. re-prefill: causal self-attention of the 32768-token context, layer by
+     layer (the R = 100 % end point of Eq. 2);
+  3. suffix redecode: 64 queries over the 34816-token spliced cache, layer by
+     layer, split-KV.
+
+The printed metric is attention TFLOP/s over the whole step (algorithmic,
+causal-visible flops 4 d Hq (R (T - R) + R (R + 1) / 2) per layer), with the
+splice GB/s (8192 algorithmic bytes per moved token-layer) beside it.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+Under torchrun every rank runs its own replica of the workload (the path
+needs no exchange step); rank 0 prints the line with the max time over ranks.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "suffix-redecode attention TFLOP/s + splice/rotate GB/s, % of GB300 roofline"
+HQ, HKV, D, PAGE = 40, 8, 128, 16
+
+
+def attn_flops(T: int, R: int, n_layers: int) -> float:
+    return 4.0 * D * HQ * (R * (T - R) + R * (R + 1) / 2.0) * n_layers
+
+
+def max_over_ranks(x: float, dist, device) -> float:
+    """Largest value of x over all ranks (identity without a process group)."""
+    if dist is None:
+        return float(x)
+    import torch
+    t = torch.tensor([float(x)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_throughput(flops_per_step_per_rank: float, world: int, ms_per_step: float) -> float:
+    """Whole-job TFLOP/s: every rank runs its own replica of the step."""
+    return world * flops_per_step_per_rank / (ms_per_step * 1e-3) / 1e12
+
+
+def measured_peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            return json.load(f), "measured"
+    except OSError:
+        return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}, "fallback"
+
+
+# ------------------------------------------------------------------ clocks
+class ClockSampler:
+    """nvidia-smi samples of SM clock and throttle reasons during the timed region."""
+
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+        self.path = os.path.join("/tmp", f"nexus_clocks_{os.getpid()}.csv")
+
+    def start(self):
+        try:
+            self.f = open(self.path, "w")
+            self.proc = subprocess.Popen(["nvidia-smi", f"--id={self.index}", f"--query-gpu={self.Q}",
+                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                         stdout=self.f, stderr=subprocess.DEVNULL)
+        except OSError:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.f.close()
+        sm, smax, power, reasons = [], [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        with open(self.path) as f:
+            for line in f:
+                parts = [p.strip() for p in line.split(",")]
+                if len(parts) < 9:
+                    continue
+                try:
+                    sm.append(float(parts[1]))
+                    smax.append(float(parts[2]))
+                    power.append(float(parts[3]))
+                except ValueError:
+                    continue
+                for n, v in zip(names, parts[5:9]):
+                    if v.lower().startswith("active"):
+                        reasons.add(n)
+        os.unlink(self.path)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
+        loaded = [s for s, p in zip(sm, power) if p > 0.5 * max(power)] or sm
+        return {"sm_mhz": statistics.median(loaded), "sm_max_mhz": max(smax),
+                "power_w_max": max(power), "samples": len(sm), "reasons": sorted(reasons)}
+
+
+# --------------------------------------------------------------- workload
+class C5:
+    """Device-resident c5 workload and the library calls of one step."""
+
+    def __init__(self, dev, n_layers=48):
+        import torch
+
+        from paper_2608_20397_gb300 import nexus
+        from paper_2608_20397_gb300.workloads import page_order, randn_bf16, workload
+
+        self.torch, self.nexus = torch, nexus
+        w = workload("c5", n_layers=n_layers)
+        self.w = w
+        s = w.sessions[0]
+        ins = s.inserts[0]
+        L = w.n_layers
+        self.L = L
+        self.n_past, self.T = s.n_past, w.spliced_len(s)
+        self.R_split = nexus.suffix_len(s.suffix_span, s.suffix_pct)
+        self.depth, self.Lb = ins.depth, ins.length
+        self.max_pages = -(-self.T // PAGE) + 1
+        n_pages = -(-self.n_past // PAGE) + self.max_pages + 16
+        self.pool = nexus.PagePool(n_pages, page_order(n_pages, w.seed, w.shuffle_pages))
+        self.kp = torch.zeros((L, n_pages, HKV, PAGE, D), dtype=torch.bfloat16, device=dev)
+        self.vp = torch.zeros_like(self.kp)
+        h_pt = np.full((2, self.max_pages), -1, np.int32)
+        npg = -(-self.n_past // PAGE)
+        h_pt[0, :npg] = self.pool.alloc(npg)
+        # live cache straight into its pages, one layer at a time (setup only)
+        pos = torch.arange(self.n_past, device=dev)
+        pg = torch.as_tensor(h_pt[0], device=dev)[pos // PAGE].long()
+        for l in range(L):
+            k = randn_bf16((1, self.n_past, HKV, D), 500 + l, dev)
+            v = randn_bf16((1, self.n_past, HKV, D), 600 + l, dev)
+            self.kp[l, pg, :, pos % PAGE] = k[0]
+            self.vp[l, pg, :, pos % PAGE] = v[0]
+        self.bk = randn_bf16((L, self.Lb, HKV, D), 700, dev)
+        self.bv = randn_bf16((L, self.Lb, HKV, D), 701, dev)
+        self.cache = nexus.kv_cache(self.kp, self.vp, n_pages, L, HKV)
+        self.blocks = [nexus.block(self.bk, self.bv, self.Lb, ins.base_pos, L, HKV)]
+        new_pt, self.segs, _ = nexus.plan_splice(self.pool, h_pt[0], self.n_past, self.max_pages,
+                                                 self.blocks, [(self.depth, 0)], 0, 1)
+        h_pt[1] = new_pt
+        self.h_pt = h_pt
+        self.d_pt = torch.as_tensor(h_pt, device=dev)
+        self.q_pre = randn_bf16((L, self.n_past, HQ, D), 800, dev)
+        self.o_pre = torch.empty_like(self.q_pre)
+        self.lse_pre = torch.empty((L, self.n_past, HQ), dtype=torch.float32, device=dev)
+        self.q_suf = randn_bf16((L, self.R_split, HQ, D), 900, dev)
+        self.o_suf = torch.empty_like(self.q_suf)
+        self.lse_suf = torch.empty((L, self.R_split, HQ), dtype=torch.float32, device=dev)
+        self.ws_bytes, self.splits = nexus.attention_workspace_size([self.T], [self.R_split], HQ, HKV,
+                                                                    1, 0)
+        self.ws = torch.empty(max(16, self.ws_bytes), dtype=torch.uint8, device=dev)
+        self.splice_rows = self.Lb + (self.n_past - self.depth)
+        self.splice_bytes = 8192.0 * self.splice_rows * L
+        self.flops_pre = attn_flops(self.n_past, self.n_past, L)
+        self.flops_suf = attn_flops(self.T, self.R_split, L)
+        self.launches_per_step = 1 + L + L * (2 if self.splits > 1 else 1)
+
+    # library calls of one step; optional events bracket the splice and the re-prefill
+    def step(self, stream, ev=None, q_pre=None, o_pre=None):
+        nexus = self.nexus
+        if ev is not None:
+            ev[0].record(stream)
+        nexus.splice_kv(self.cache, self.d_pt, None, 2, self.max_pages, self.blocks, self.segs, 0,
+                        self.L, stream)
+        if ev is not None:
+            ev[1].record(stream)
+        for l in range(self.L):
+            nexus.reprefill(self.cache, self.d_pt, 2, self.max_pages, [self.n_past],
+                            self.q_pre[l:l + 1] if q_pre is None else q_pre(l),
+                            self.o_pre[l:l + 1] if o_pre is None else o_pre(l),
+                            self.lse_pre[l:l + 1], HQ, l, l + 1, rows=[0], split_kv=1,
+                            stream=stream)
+        if ev is not None:
+            ev[2].record(stream)
+        for l in range(self.L):
+            nexus.suffix_attention(self.cache, self.d_pt, 2, self.max_pages, [self.T],
+                                   [self.R_split], self.q_suf[l:l + 1], self.o_suf[l:l + 1],
+                                   self.lse_suf[l:l + 1], HQ, l, l + 1, rows=[1], split_kv=0,
+                                   workspace=self.ws, workspace_bytes=self.ws_bytes, stream=stream)
+        if ev is not None:
+            ev[3].record(stream)
+
+
+# ----------------------------------------------------------- cpu baseline
+def oracle_sample_timing(q_rows, k, v, live_k, bk, n_rows_target_s=10.0, max_rows=64):
+    """Times the fp64 oracle on a bounded sample of the same workload and
+    returns (TFLOP/s, GB/s, description): attention rows of the re-prefill at
+    the deep end of the context, and a splice of 64 block rows of one layer."""
+    import oracle
+    T = k.shape[0]
+    flops, t_attn, rows_done = 0.0, 0.0, 0
+    while rows_done < max_rows and t_attn < n_rows_target_s:
+        r = min(4, max_rows - rows_done)
+        pos = np.arange(T - r, T) - 4 * (rows_done // 4)
+        t0 = time.perf_counter()
+        oracle.attention(q_rows[rows_done:rows_done + r], k, v, pos, HQ // HKV)
+        t_attn += time.perf_counter() - t0
+        flops += sum(4.0 * D * HQ * (p + 1) for p in pos)
+        rows_done += r
+    t0 = time.perf_counter()
+    oracle.splice_sequence(live_k, live_k, [(live_k.shape[1], bk, bk, 0)])
+    t_spl = time.perf_counter() - t0
+    spl_bytes = 8192.0 * bk.shape[1] * bk.shape[0]
+    desc = (f"fp64 NumPy oracle: {rows_done} re-prefill query rows x {HQ} heads over ~{T} keys "
+            f"(layer 0), and a {bk.shape[1]}-row block splice of one layer")
+    return flops / t_attn / 1e12, spl_bytes / t_spl / 1e9, desc, t_attn + t_spl
+
+
+def cpu_cores():
+    try:
+        return len(os.sched_getaffinity(0))
+    except AttributeError:
+        return os.cpu_count()
+
+
+def run_reference(args):
+    """Reference arm: the fp64 oracle as it stands, on the host cores, on a
+    bounded sample of the c5 workload per step."""
+    import torch
+
+    from paper_2608_20397_gb300.workloads import randn_bf16
+    f64 = lambda t: t.float().double().numpy()
+    T = 32768
+    k = f64(randn_bf16((T, HKV, D), 500, "cpu"))
+    v = f64(randn_bf16((T, HKV, D), 600, "cpu"))
+    q = f64(randn_bf16((64, HQ, D), 800, "cpu"))
+    bk = f64(randn_bf16((1, 64, HKV, D), 700, "cpu"))
+    live = f64(randn_bf16((1, 64, HKV, D), 501, "cpu"))
+    vals, times, desc = [], [], ""
+    for i in range(args.warmup + args.steps):
+        t0 = time.perf_counter()
+        tf, gbs, desc, _ = oracle_sample_timing(q, k, v, live, bk, n_rows_target_s=4.0, max_rows=16)
+        dt = time.perf_counter() - t0
+        if i >= args.warmup:
+            vals.append(tf)
+            times.append(dt)
+    value = statistics.median(vals)
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "TFLOP/s",
+            "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": 1e3 * statistics.median(times), "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": "c5 deep-context (bounded oracle sample per step)"},
+            "cpu_baseline": {"value": value, "unit": "TFLOP/s", "cores": cpu_cores(),
+                             "kind": "oracle", "sample": desc},
+            "e2e": {"value": value, "unit": "TFLOP/s", "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+# ------------------------------------------------------------------- main
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=5)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--layers", type=int, default=48, help="layers of the workload (48 = c5)")
+    ap.add_argument("--profile", choices=["reprefill", "splice", "suffix"], default=None,
+                    help="run only this kernel of the step (small case for ncu captures)")
+    args = ap.parse_args()
+
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    if args.impl == "reference":
+        if rank == 0:
+            run_reference(args)
+        return
+
+    import torch
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=dev)
+
+    from paper_2608_20397_gb300 import nexus
+    nexus.lib()
+    wl = C5(dev, args.layers)
+    stream = torch.cuda.current_stream()
+    peaks, peak_kind = measured_peaks()
+
+    def barrier():
+        if dist is not None:
+            dist.barrier()
+        torch.cuda.synchronize()
+
+    if args.profile:
+        _profile_only(wl, args, stream)
+        return
+
+    for _ in range(args.warmup):
+        wl.step(stream)
+    st = nexus.device_status(stream)
+    if st != nexus.OK:
+        raise RuntimeError(f"device status after warm-up: {nexus.status_string(st)}")
+
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(args.steps)]
+    sampler = ClockSampler(dev.index)
+    sampler.start()
+    time.sleep(0.5)
+    barrier()
+    t_start = torch.cuda.Event(enable_timing=True)
+    t_end = torch.cuda.Event(enable_timing=True)
+    t_start.record(stream)
+    for i in range(args.steps):
+        wl.step(stream, evs[i])
+    t_end.record(stream)
+    barrier()
+    clocks = sampler.stop()
+    st = nexus.device_status(stream)
+    if st != nexus.OK:
+        raise RuntimeError(f"device status after timed steps: {nexus.status_string(st)}")
+    total_ms = t_start.elapsed_time(t_end)
+    splice_ms = statistics.mean(e[0].elapsed_time(e[1]) for e in evs)
+    pre_ms = statistics.mean(e[1].elapsed_time(e[2]) for e in evs)
+    suf_ms = statistics.mean(e[2].elapsed_time(e[3]) for e in evs)
+    total_ms = max_over_ranks(total_ms, dist, dev)
+    ms_per_step = total_ms / args.steps
+    flops_step = wl.flops_pre + wl.flops_suf
+    value = job_throughput(flops_step, world, ms_per_step)
+
+    pre_launch_s = pre_ms * 1e-3 / wl.L
+    achieved = (wl.flops_pre / wl.L) / pre_launch_s / 1e12
+    peak_tc = peaks.get("bf16_tflops_sustained", peaks["bf16_tflops"])
+    traffic = _profiled_traffic("attention_kernel")
+    roofline = {"bound": "tensor", "kernel": "attention_kernel (re-prefill, one layer per launch)",
+                "achieved": achieved, "peak": peak_tc, "unit": "TFLOP/s",
+                "frac": achieved / peak_tc, "peak_kind": f"bf16 sustained, {peak_kind}",
+                "traffic": traffic}
+    splice_gbs = wl.splice_bytes / (splice_ms * 1e-3) / 1e9
+    roofline_splice = {"bound": "hbm", "kernel": "splice_kernel", "achieved": splice_gbs,
+                       "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                       "frac": splice_gbs / peaks["hbm_gbs"], "peak_kind": f"copy, {peak_kind}",
+                       "frac_of_8tbs_spec": splice_gbs / 8000.0,
+                       "traffic": _profiled_traffic("splice_kernel")}
+    suf_tflops = wl.flops_suf / (suf_ms * 1e-3) / 1e12
+
+    e2e = None
+    if not args.no_e2e:
+        e2e = _e2e(wl, stream, args, barrier, world, dist, dev)
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        f64 = lambda t: t.float().cpu().double().numpy()
+        pos = torch.arange(wl.n_past, device=dev)
+        pg = wl.d_pt[0][pos // PAGE].long()
+        k0 = f64(wl.kp[0, pg, :, pos % PAGE])
+        v0 = f64(wl.vp[0, pg, :, pos % PAGE])
+        tf, gbs, desc, secs = oracle_sample_timing(f64(wl.q_pre[0, -64:]), k0, v0,
+                                                   k0[None, :64], f64(wl.bk[:1, :64]))
+        cpu = {"value": tf, "unit": "TFLOP/s", "cores": cpu_cores(), "kind": "oracle",
+               "sample": desc, "splice_gbs": gbs, "seconds": secs}
+
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": value, "unit": "TFLOP/s", "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_per_step,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+            "data": "synthetic",
+            "config": {"workload": f"c5 deep-context: {wl.L} layers, n_past {wl.n_past}, "
+                                   f"{wl.Lb}-token block at {wl.depth} (T={wl.T}); re-prefill "
+                                   f"{wl.n_past}x{wl.n_past} causal + {wl.R_split}-query "
+                                   f"split-KV suffix ({wl.splits} splits), 40/8 heads, d=128",
+                       "parallelism": f"replicas x{world}",
+                       "l2": "inputs exceed L2 (>30 GB touched per step); no flush"},
+            "splice_gbs": splice_gbs, "splice_ms": splice_ms, "reprefill_ms": pre_ms,
+            "suffix_ms": suf_ms, "suffix_tflops": suf_tflops,
+            "roofline": roofline, "roofline_splice": roofline_splice,
+            "e2e": e2e, "cpu_baseline": cpu, "clocks": clocks,
+            "gpu_launches": wl.launches_per_step * args.steps,
+        }
+        print(json.dumps(line), flush=True)
+    if dist is not None:
+        dist.destroy_process_group()
+
+
+def _profile_only(wl, args, stream):
+    """W + K launches of one kernel of the step on the (reduced) workload,
+    for ncu captures; prints the mean CUDA-event time per launch."""
+    import torch
+    nexus = wl.nexus
+
+    def one():
+        if args.profile == "splice":
+            nexus.splice_kv(wl.cache, wl.d_pt, None, 2, wl.max_pages, wl.blocks, wl.segs, 0, wl.L,
+                            stream)
+        elif args.profile == "reprefill":
+            nexus.reprefill(wl.cache, wl.d_pt, 2, wl.max_pages, [wl.n_past], wl.q_pre[:1],
+                            wl.o_pre[:1], wl.lse_pre[:1], HQ, 0, 1, rows=[0], split_kv=1,
+                            stream=stream)
+        else:
+            nexus.suffix_attention(wl.cache, wl.d_pt, 2, wl.max_pages, [wl.T], [wl.R_split],
+                                   wl.q_suf[:1], wl.o_suf[:1], wl.lse_suf[:1], HQ, 0, 1, rows=[1],
+                                   split_kv=0, workspace=wl.ws, workspace_bytes=wl.ws_bytes,
+                                   stream=stream)
+
+    for _ in range(args.warmup):
+        one()
+    torch.cuda.synchronize()
+    a = torch.cuda.Event(enable_timing=True)
+    b = torch.cuda.Event(enable_timing=True)
+    a.record(stream)
+    for _ in range(args.steps):
+        one()
+    b.record(stream)
+    torch.cuda.synchronize()
+    st = nexus.device_status(stream)
+    print(json.dumps({"profile": args.profile, "layers": wl.L, "ms_per_launch":
+                      a.elapsed_time(b) / args.steps, "status": nexus.status_string(st)}), flush=True)
+    if st != nexus.OK:
+        raise SystemExit(1)
+
+
+def _profiled_traffic(kernel: str):
+    """DRAM bytes (read + write) per launch from the committed ncu summary, or
+    None when there is none or the kernel source changed since the capture."""
+    import hashlib
+    path = os.path.join(ROOT, "profiles", "traffic.json")
+    try:
+        with open(path) as f:
+            entry = json.load(f).get(kernel)
+        if not entry:
+            return None
+        with open(os.path.join(ROOT, entry["source"]), "rb") as f:
+            if hashlib.sha256(f.read()).hexdigest() != entry["source_sha256"]:
+                return None
+        return entry["bytes_per_launch"]
+    except (OSError, ValueError, KeyError):
+        return None
+
+
+def _e2e(wl, stream, args, barrier, world, dist, dev):
+    """The same step through the C ABI with host buffers: every step copies the
+    block K/V and every layer's Q from pinned host memory and reads every
+    layer's O back, inside the timed region."""
+    import torch
+    L = wl.L
+    h_bk = torch.empty(wl.bk.shape, dtype=torch.bfloat16, pin_memory=True)
+    h_bv = torch.empty(wl.bv.shape, dtype=torch.bfloat16, pin_memory=True)
+    h_bk.copy_(wl.bk)
+    h_bv.copy_(wl.bv)
+    h_q = torch.empty(wl.q_pre.shape[1:], dtype=torch.bfloat16, pin_memory=True)
+    h_o = torch.empty(wl.o_pre.shape[1:], dtype=torch.bfloat16, pin_memory=True)
+    h_qs = torch.empty(wl.q_suf.shape, dtype=torch.bfloat16, pin_memory=True)
+    h_os = torch.empty(wl.o_suf.shape, dtype=torch.bfloat16, pin_memory=True)
+    h_q.copy_(wl.q_pre[0])
+    h_qs.copy_(wl.q_suf)
+    qbuf = torch.empty_like(wl.q_pre[:1])
+    obuf = torch.empty_like(wl.o_pre[:1])
+    h2d = (h_bk.numel() + h_bv.numel() + L * h_q.numel() + h_qs.numel()) * 2
+    d2h = (L * h_o.numel() + h_os.numel()) * 2
+
+    def one():
+        wl.bk.copy_(h_bk, non_blocking=True)
+        wl.bv.copy_(h_bv, non_blocking=True)
+        wl.q_suf.copy_(h_qs, non_blocking=True)
+
+        nexus = wl.nexus
+        nexus.splice_kv(wl.cache, wl.d_pt, wl.h_pt, 2, wl.max_pages, wl.blocks, wl.segs, 0, L,
+                        stream)
+        for l in range(L):
+            qbuf[0].copy_(h_q, non_blocking=True)
+            nexus.reprefill(wl.cache, wl.d_pt, 2, wl.max_pages, [wl.n_past], qbuf, obuf,
+                            wl.lse_pre[l:l + 1], HQ, l, l + 1, rows=[0], split_kv=1, stream=stream)
+            h_o.copy_(obuf[0], non_blocking=True)
+        for l in range(L):
+            nexus.suffix_attention(wl.cache, wl.d_pt, 2, wl.max_pages, [wl.T], [wl.R_split],
+                                   wl.q_suf[l:l + 1], wl.o_suf[l:l + 1], wl.lse_suf[l:l + 1], HQ,
+                                   l, l + 1, rows=[1], split_kv=0, workspace=wl.ws,
+                                   workspace_bytes=wl.ws_bytes, stream=stream)
+        h_os.copy_(wl.o_suf, non_blocking=True)
+
+    for _ in range(max(1, min(args.warmup, 2))):
+        one()
+    barrier()
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        one()
+    barrier()
+    secs = max_over_ranks(time.perf_counter() - t0, dist, dev)
+    per = secs / args.steps
+    flops = wl.flops_pre + wl.flops_suf
+    return {"value": job_throughput(flops, world, per * 1e3), "unit": "TFLOP/s",
+            "ms_per_step": per * 1e3,
+            "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h)}
+
+
+if __name__ == "__main__":
+    main()

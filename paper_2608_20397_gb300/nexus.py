@@ -239,16 +239,20 @@ class PagePool:
 def kv_cache(k_pool, v_pool, n_pages: int, n_layers: int, n_kv_heads: int = 8,
              v_transposed: bool = False, rope_type: int = ROPE_NEOX, rope_theta: float = 1.0e6,
              rope_freq_scale: float = 1.0) -> KvCache:
-    return KvCache(_ptr(k_pool), _ptr(v_pool), int(n_pages), int(n_layers), int(n_kv_heads), 128,
-                   16, int(bool(v_transposed)), int(rope_type), float(rope_theta),
-                   float(rope_freq_scale))
+    c = KvCache(_ptr(k_pool), _ptr(v_pool), int(n_pages), int(n_layers), int(n_kv_heads), 128,
+                16, int(bool(v_transposed)), int(rope_type), float(rope_theta),
+                float(rope_freq_scale))
+    c._keep = (k_pool, v_pool)   # the descriptor holds raw pointers: keep the buffers alive
+    return c
 
 
 def block(k, v, n_tokens: int, base_pos: int, n_layers: int, n_kv_heads: int = 8,
           rope_type: int = ROPE_NEOX, rope_theta: float = 1.0e6,
           rope_freq_scale: float = 1.0) -> Block:
-    return Block(_ptr(k), _ptr(v), int(n_tokens), int(base_pos), int(n_layers), int(n_kv_heads),
-                 128, int(rope_type), float(rope_theta), float(rope_freq_scale))
+    b = Block(_ptr(k), _ptr(v), int(n_tokens), int(base_pos), int(n_layers), int(n_kv_heads),
+              128, int(rope_type), float(rope_theta), float(rope_freq_scale))
+    b._keep = (k, v)
+    return b
 
 
 def segments_array(segs) -> ctypes.Array:
