@@ -309,6 +309,32 @@ size_t nexus_attention_workspace_size(int32_t n_seqs, const int32_t* h_kv_len,
                                       int32_t n_kv_heads, int32_t n_layers_call,
                                       int32_t split_kv, int32_t* splits_out);
 
+/* ------------------------------------------------ attention, no allocation */
+/* nexus_suffix_attention for callers that cannot allocate device memory: code
+ * running while a stream is captured (no cudaMalloc there), plug-ins handed only
+ * their input and output buffers, or processes with a fixed memory pool. The
+ * paper has no counterpart; this is a deployment convenience of this library.
+ *
+ * Arguments, results and errors are those of nexus_suffix_attention, without
+ * the workspace: the split-KV partials live in a 32 MiB array inside the
+ * library, which every GPU that loads the library holds until the process
+ * exits. Requests whose partials need more than 32 MiB (see
+ * nexus_attention_workspace_size) return NEXUS_ENOMEM before any launch; pass
+ * split_kv = 1 to need none. The first call on each device looks up the array's
+ * device address with that device current; make that first call before any
+ * stream capture. Every call shares the one array and overwrites what the
+ * previous call left (nothing in it needs to start at zero), so calls that may
+ * run at the same time on the GPU (different streams, no ordering between
+ * them) race; order them on one stream or with events. Allocates nothing. */
+nexus_status nexus_suffix_attention_noalloc(const nexus_kv_cache* cache,
+                                            const int32_t* d_page_tables, int32_t n_rows,
+                                            int32_t max_pages, int32_t n_seqs,
+                                            const int32_t* h_rows, const int32_t* h_kv_len,
+                                            const int32_t* h_q_len, const void* q, void* out,
+                                            float* lse, int32_t n_q_heads, int32_t layer_begin,
+                                            int32_t layer_end, int32_t split_kv,
+                                            nexus_stream stream);
+
 #ifdef __cplusplus
 }
 #endif

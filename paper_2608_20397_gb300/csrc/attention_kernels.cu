@@ -20,6 +20,8 @@
 // drains its in-flight copies and MMAs, frees TMEM and exits.
 #include <cuda_bf16.h>
 
+#include <mutex>
+
 #include "internal.h"
 #include "ptx.cuh"
 
@@ -523,3 +525,63 @@ cudaError_t attention_take_timeout(unsigned int* flag, cudaStream_t stream) {
 }
 
 }  // namespace nexus
+
+// ---------------------------------------------------------------------------
+// Attention without any device allocation by the caller.
+//
+// Some callers cannot obtain device memory for the split-KV partials: code
+// running while a stream is being captured (cudaMalloc is not allowed there),
+// plug-ins that only ever receive their input and output buffers from a host
+// framework, or processes whose memory pool is fixed up front. For them the
+// partials live in one file-scope array that the module owns; every GPU that
+// loads this library keeps it until the process exits.
+// ---------------------------------------------------------------------------
+namespace nexus {
+namespace {
+constexpr size_t kStaticScratchBytes = size_t(32) << 20;   // 32 MiB
+static __device__ __align__(256) unsigned char g_static_split_scratch[kStaticScratchBytes];
+
+constexpr int kMaxScratchDevices = 64;
+std::mutex g_scratch_mu;
+void* g_scratch_addr[kMaxScratchDevices] = {};
+
+// Device address of the array on the current device. Host code cannot use the
+// array's name as a device pointer, so the address is looked up once per
+// device (with that device current) and remembered.
+cudaError_t static_scratch_address(void** out) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (dev < 0 || dev >= kMaxScratchDevices) return cudaErrorInvalidDevice;
+  std::lock_guard<std::mutex> lock(g_scratch_mu);
+  if (!g_scratch_addr[dev]) {
+    void* p = nullptr;
+    e = cudaGetSymbolAddress(&p, g_static_split_scratch);
+    if (e != cudaSuccess) return e;
+    g_scratch_addr[dev] = p;
+  }
+  *out = g_scratch_addr[dev];
+  return cudaSuccess;
+}
+}  // namespace
+}  // namespace nexus
+
+extern "C" nexus_status nexus_suffix_attention_noalloc(
+    const nexus_kv_cache* cache, const int32_t* d_page_tables, int32_t n_rows, int32_t max_pages,
+    int32_t n_seqs, const int32_t* h_rows, const int32_t* h_kv_len, const int32_t* h_q_len,
+    const void* q, void* out, float* lse, int32_t n_q_heads, int32_t layer_begin,
+    int32_t layer_end, int32_t split_kv, nexus_stream stream) {
+  if (!cache) return NEXUS_EINVAL;
+  const size_t need = nexus_attention_workspace_size(n_seqs, h_kv_len, h_q_len, n_q_heads,
+                                                     cache->n_kv_heads, layer_end - layer_begin,
+                                                     split_kv, nullptr);
+  if (need > nexus::kStaticScratchBytes) return NEXUS_ENOMEM;
+  void* scratch = nullptr;
+  if (nexus::static_scratch_address(&scratch) != cudaSuccess) {
+    cudaGetLastError();
+    return NEXUS_ECUDA;
+  }
+  return nexus_suffix_attention(cache, d_page_tables, n_rows, max_pages, n_seqs, h_rows, h_kv_len,
+                                h_q_len, q, out, lse, n_q_heads, layer_begin, layer_end, split_kv,
+                                scratch, nexus::kStaticScratchBytes, stream);
+}

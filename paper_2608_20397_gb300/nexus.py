@@ -106,6 +106,10 @@ _SIGS = {
                                   c_int32, c_void_p, c_size_t, c_void_p]),
     "nexus_attention_workspace_size": (c_size_t, [c_int32, _i32p, _i32p, c_int32, c_int32,
                                                   c_int32, c_int32, _i32p]),
+    "nexus_suffix_attention_noalloc": (c_int32, [POINTER(KvCache), c_void_p, c_int32, c_int32,
+                                                 c_int32, _i32p, _i32p, _i32p, c_void_p,
+                                                 c_void_p, c_void_p, c_int32, c_int32, c_int32,
+                                                 c_int32, c_void_p]),
 }
 EXPORTED = tuple(_SIGS)
 
@@ -361,3 +365,17 @@ def reprefill(cache: KvCache, d_page_tables, n_rows: int, max_pages: int, kv_len
 def device_status(stream=None) -> int:
     """Synchronises the stream; OK, ETIMEOUT (a bounded device wait gave up) or ECUDA."""
     return int(lib().nexus_device_status(_stream(stream)))
+
+
+def suffix_attention_noalloc(cache: KvCache, d_page_tables, n_rows: int, max_pages: int, kv_len,
+                             q_len, q, out, lse=None, n_q_heads: int = 40, layer_begin: int = 0,
+                             layer_end: int = 1, rows=None, split_kv: int = 0, stream=None):
+    """nexus_suffix_attention for callers that cannot allocate device memory:
+    the split partials use the library's own 32 MiB array (see nexus.h)."""
+    kv = _i32(kv_len)
+    ql = _i32(q_len)
+    rw = _i32(rows)
+    _check("nexus_suffix_attention_noalloc", lib().nexus_suffix_attention_noalloc(
+        ctypes.byref(cache), _ptr(d_page_tables), int(n_rows), int(max_pages), len(kv[1]),
+        rw[0] if rw else None, kv[0], ql[0], _ptr(q), _ptr(out), _ptr(lse), int(n_q_heads),
+        int(layer_begin), int(layer_end), int(split_kv), _stream(stream)))
