@@ -2,22 +2,30 @@
 // (softmax(QK^T / sqrt(d)) V of Sec. III-A over the redecoded suffix of
 // Sec. III-C / Sec. V-A), plus the split-KV partial merge.
 //
-// One CTA owns one 128-row query tile of one KV head: rows are (token, head in
-// the GQA group) pairs, 128 / group tokens x group heads, so every K/V tile
-// brought into shared memory serves all query heads that read it. Per CTA:
+// One CTA owns two 128-row query tiles (A and B) of one KV head. Rows are
+// (token, head in the GQA group) pairs, 128 / group tokens x group heads, so
+// every K/V tile brought into shared memory serves all query heads that read
+// it, twice. Per CTA (320 threads):
 //
-//   warp 4    TMA producer: the Q tile once, then K and V tiles of 128 keys
-//             (eight 16-token pages each, fetched through the page table)
-//             into a two-stage ring
-//   warp 5    MMA issuer: S = Q K^T into TMEM (double-buffered), then
-//             O += P V into TMEM, with tcgen05.mma (bf16 in, f32 accumulate)
-//   warps 0-3 softmax: thread i owns TMEM lane i (= tile row i); online
-//             softmax in the log2 domain with a lazily moved running max,
-//             P written to shared memory as bf16, final O / l and LSE
+//   warp 8     TMA producer: both Q tiles once, then K and V tiles of 128 keys
+//              (eight 16-token pages each, through the page table) into a
+//              two-stage ring
+//   warp 9     MMA issuer (tcgen05.mma, bf16 in, f32 accumulate in TMEM):
+//              S_A(0) S_B(0), then per key tile j:
+//              PV_A(j) S_A(j+1) PV_B(j) S_B(j+1)
+//              so the tensor core always has two products queued while one
+//              softmax warpgroup works
+//   warps 0-3  softmax of tile A, warps 4-7 softmax of tile B: thread i of a
+//              warpgroup owns TMEM lane i (= tile row i); online softmax in the
+//              log2 domain, the running max moved only past 2^8 growth (then O
+//              is rescaled in TMEM); P is written back as bf16 over the first 64
+//              columns of the tile's own S and read from TMEM by the P V product
 //
-// TMEM columns: S0 [0,128), S1 [128,256), O [256,384) of a 512-column
-// allocation. Every wait is bounded; on expiry the CTA records a timeout,
-// drains its in-flight copies and MMAs, frees TMEM and exits.
+// TMEM columns: S_A [0,128), S_B [128,256), O_A [256,384), O_B [384,512).
+// The S-full barrier of tile X at step j is committed after PV_X(j-1), so it
+// also certifies that O_X and the P columns are free. Every wait is bounded;
+// on expiry the CTA records a timeout, drains its in-flight copies and MMAs,
+// frees TMEM and exits.
 #include <cuda_bf16.h>
 
 #include <mutex>
@@ -36,29 +44,27 @@ constexpr int BM = 128;   // query rows per tile
 constexpr int BN = 128;   // keys per tile
 constexpr int D = kHeadDim;
 constexpr int kStages = 2;
-constexpr int kThreads = 192;
-constexpr int kProducerWarp = 4;
-constexpr int kMmaWarp = 5;
+constexpr int kThreads = 320;
+constexpr int kProducerWarp = 8;
+constexpr int kMmaWarp = 9;
 constexpr uint32_t kTileBytes = BM * D * 2;   // 32 KiB
 constexpr uint32_t kHalf = 16384;             // one 64-column half of a tile
 constexpr uint64_t kBudgetNs = 2000000000ull; // 2 s per wait
 constexpr uint64_t kDrainNs = 200000000ull;   // 0.2 s to drain after an abort
 constexpr float kRescaleThreshold = 8.0f;     // move the running max only past 2^8 growth
 
-constexpr uint32_t OFF_Q = 0;
-constexpr uint32_t OFF_K = OFF_Q + kTileBytes;
+constexpr uint32_t OFF_Q = 0;                          // tile A, tile B
+constexpr uint32_t OFF_K = OFF_Q + 2 * kTileBytes;
 constexpr uint32_t OFF_V = OFF_K + kStages * kTileBytes;
-constexpr uint32_t OFF_P = OFF_V + kStages * kTileBytes;
-constexpr uint32_t OFF_BAR = OFF_P + kTileBytes;
+constexpr uint32_t OFF_BAR = OFF_V + kStages * kTileBytes;
 enum {
   B_Q = 0,
   B_KF = 1,      // +stage
   B_VF = 3,      // +stage
   B_KVE = 5,     // +stage
-  B_SF = 7,      // +buffer
-  B_SFREE = 9,   // +buffer
-  B_PF = 11,
-  B_OD = 12,
+  B_SF = 7,      // +tile
+  B_PF = 9,      // +tile
+  B_OD = 11,     // +tile
   B_FIN = 13,
   kNumBars = 14
 };
@@ -66,48 +72,55 @@ constexpr uint32_t OFF_MISC = OFF_BAR + kNumBars * 8;
 constexpr uint32_t kSmemUsed = OFF_MISC + 16;
 constexpr uint32_t kSmemBytes = kSmemUsed + 1024;   // slack for 1024-byte alignment
 
-constexpr uint32_t TM_S0 = 0, TM_O = 256;
+constexpr uint32_t TM_S = 0;     // + 128 * tile
+constexpr uint32_t TM_O = 256;   // + 128 * tile
 
 __device__ __forceinline__ void record_timeout(volatile int* abort) {
   *abort = 1;
   atomicOr(&g_attn_timeout, 1u);
 }
 
-struct Tile {
-  int seq, qt, kv, layer_rel, split;
-  int tok0, ntok, pos0, kt_begin, n_tiles;
+struct Work {
+  int seq, kv, layer_rel, split;
+  int tok0[2], ntok[2], pos0[2];
+  bool has_b;
+  int kt_begin, n_tiles;
 };
 
-__device__ __forceinline__ Tile decode_tile(const AttnLaunch& p) {
-  Tile t;
+__device__ __forceinline__ Work decode_work(const AttnLaunch& p) {
+  Work w;
   const int rev = p.total_tiles - 1 - (int)blockIdx.x;   // deepest query tiles first
   int lo = 0, hi = p.n_seqs - 1;
   while (lo < hi) {
     const int mid = (lo + hi + 1) >> 1;
     if (p.tile_prefix[mid] <= rev) lo = mid; else hi = mid - 1;
   }
-  t.seq = lo;
-  t.qt = rev - p.tile_prefix[lo];
-  t.kv = blockIdx.y;
-  t.layer_rel = blockIdx.z / p.splits;
-  t.split = blockIdx.z % p.splits;
+  w.seq = lo;
+  const int pair = rev - p.tile_prefix[lo];
+  w.kv = blockIdx.y;
+  w.layer_rel = blockIdx.z / p.splits;
+  w.split = blockIdx.z % p.splits;
   const AttnSeq& s = p.seq[lo];
-  t.tok0 = t.qt * p.tile_tokens;
-  t.ntok = min(p.tile_tokens, s.q_len - t.tok0);
-  t.pos0 = s.kv_len - s.q_len + t.tok0;
-  const int pos_last = t.pos0 + t.ntok - 1;
+  const int q_tiles = (s.q_len + p.tile_tokens - 1) / p.tile_tokens;
+  w.has_b = 2 * pair + 1 < q_tiles;
+  for (int x = 0; x < 2; ++x) {
+    w.tok0[x] = (2 * pair + x) * p.tile_tokens;
+    w.ntok[x] = max(0, min(p.tile_tokens, s.q_len - w.tok0[x]));
+    w.pos0[x] = s.kv_len - s.q_len + w.tok0[x];
+  }
+  const int last = w.has_b ? 1 : 0;
+  const int pos_last = w.pos0[last] + w.ntok[last] - 1;
   const int kt_total = pos_last / BN + 1;
   const int per = (kt_total + p.splits - 1) / p.splits;
-  t.kt_begin = t.split * per;
-  t.n_tiles = max(0, min(kt_total, t.kt_begin + per) - t.kt_begin);
-  return t;
+  w.kt_begin = w.split * per;
+  w.n_tiles = max(0, min(kt_total, w.kt_begin + per) - w.kt_begin);
+  return w;
 }
 
 // Zeroes V rows of keys [r0, 128) of one stage, so cache slots past kv_len
 // (whatever bits they hold) contribute exactly 0 to P V.
 __device__ __forceinline__ void zero_v_rows(uint8_t* vbuf, int r0, bool vt, int lane) {
   if (!vt) {
-    // two halves of [128 keys][128 B]
     for (int i = lane; i < 2 * (BN - r0) * 8; i += 32) {
       const int half = i / ((BN - r0) * 8);
       const int rem = i % ((BN - r0) * 8);
@@ -130,6 +143,43 @@ __device__ __forceinline__ void zero_v_rows(uint8_t* vbuf, int r0, bool vt, int 
   }
 }
 
+__device__ __forceinline__ float fmax3(float a, float b, float c) {
+  float d;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
+  return d;
+}
+
+// D[tmem] (+)= A[tmem] * B[smem]: A is read from tensor memory (P, packed
+// bf16 pairs along K, row i in lane i).
+__device__ __forceinline__ void mma_bf16_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t b_desc,
+                                            uint32_t idesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n"
+      " .reg .pred p;\n"
+      " setp.ne.b32 p, %4, 0;\n"
+      " tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n"
+      "}\n" ::"r"(d_tmem),
+      "r"(a_tmem), "l"(b_desc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+
+__device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t (&r)[16]) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], "
+      "{%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16};" ::"r"(taddr),
+      "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]),
+      "r"(r[8]), "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]),
+      "r"(r[15])
+      : "memory");
+}
+
+__device__ __forceinline__ void tmem_st8(uint32_t taddr, const uint32_t (&r)[8]) {
+  asm volatile("tcgen05.st.sync.aligned.32x32b.x8.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8};" ::"r"(taddr),
+               "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]),
+               "r"(r[7])
+               : "memory");
+}
+
 __global__ void __launch_bounds__(kThreads, 1)
 attention_kernel(const __grid_constant__ AttnLaunch p, const __grid_constant__ AttnMaps maps) {
   extern __shared__ uint8_t smem_raw[];
@@ -144,19 +194,22 @@ attention_kernel(const __grid_constant__ AttnLaunch p, const __grid_constant__ A
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
-  const Tile t = decode_tile(p);
-  const AttnSeq sq = p.seq[t.seq];
+  const Work w = decode_work(p);
+  const AttnSeq sq = p.seq[w.seq];
   const int G = p.group;
-  const int layer = p.layer_begin + t.layer_rel;
+  const int layer = p.layer_begin + w.layer_rel;
+  const int n_tiles = w.n_tiles;
+  const int n_q = w.has_b ? 2 : 1;
 
   // ---- setup: zero the Q rows no TMA box writes, init barriers, alloc TMEM
   {
     const int rows_loaded = G * p.tile_tokens;
-    for (int i = threadIdx.x; i < 2 * (BM - rows_loaded) * 8; i += kThreads) {
-      const int half = i / ((BM - rows_loaded) * 8);
-      const int rem = i % ((BM - rows_loaded) * 8);
-      reinterpret_cast<uint4*>(smem + OFF_Q + half * kHalf + (rows_loaded + rem / 8) * 128)[rem % 8] =
-          make_uint4(0, 0, 0, 0);
+    const int per_half = (BM - rows_loaded) * 8;
+    for (int i = threadIdx.x; i < 4 * per_half; i += kThreads) {
+      const int qh = i / per_half;   // tile * 2 + half
+      const int rem = i % per_half;
+      reinterpret_cast<uint4*>(smem + OFF_Q + (qh >> 1) * kTileBytes + (qh & 1) * kHalf +
+                               (rows_loaded + rem / 8) * 128)[rem % 8] = make_uint4(0, 0, 0, 0);
     }
     fence_proxy_async_smem();
   }
@@ -167,12 +220,11 @@ attention_kernel(const __grid_constant__ AttnLaunch p, const __grid_constant__ A
       mbar_init(bar(B_VF + s), 1);
       mbar_init(bar(B_KVE + s), 1);
     }
-    for (int b = 0; b < 2; ++b) {
-      mbar_init(bar(B_SF + b), 1);
-      mbar_init(bar(B_SFREE + b), 128);
+    for (int x = 0; x < 2; ++x) {
+      mbar_init(bar(B_SF + x), 1);
+      mbar_init(bar(B_PF + x), 128);
+      mbar_init(bar(B_OD + x), 1);
     }
-    mbar_init(bar(B_PF), 128);
-    mbar_init(bar(B_OD), 1);
     mbar_init(bar(B_FIN), 1);
     *abort = 0;
     *never = 0;
@@ -186,9 +238,7 @@ attention_kernel(const __grid_constant__ AttnLaunch p, const __grid_constant__ A
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
-
   const bool vt = p.v_transposed != 0;
-  const int n_tiles = t.n_tiles;
 
   if (warp == kProducerWarp) {
     // ------------------------------------------------------ TMA producer
@@ -200,10 +250,11 @@ attention_kernel(const __grid_constant__ AttnLaunch p, const __grid_constant__ A
         prefetch_tmap(&maps.q);
         prefetch_tmap(&maps.k);
         prefetch_tmap(&maps.v);
-        mbar_arrive_expect_tx(bar(B_Q), 2u * G * p.tile_tokens * 128u);
-        for (int half = 0; half < 2; ++half)
-          tma_load_4d(sbase + OFF_Q + half * kHalf, &maps.q, bar(B_Q), half * 64, t.kv * G,
-                      sq.q_off + t.tok0, t.layer_rel);
+        mbar_arrive_expect_tx(bar(B_Q), 2u * n_q * G * p.tile_tokens * 128u);
+        for (int x = 0; x < n_q; ++x)
+          for (int half = 0; half < 2; ++half)
+            tma_load_4d(sbase + OFF_Q + x * kTileBytes + half * kHalf, &maps.q, bar(B_Q),
+                        half * 64, w.kv * G, sq.q_off + (x ? w.tok0[1] : w.tok0[0]), w.layer_rel);
       }
       for (int it = 0; it < n_tiles; ++it) {
         const int st = it & 1;
@@ -212,7 +263,7 @@ attention_kernel(const __grid_constant__ AttnLaunch p, const __grid_constant__ A
           ok = __all_sync(0xffffffffu, ok);
           if (!ok) { if (lane == 0) record_timeout(abort); break; }
         }
-        const int kt = t.kt_begin + it;
+        const int kt = w.kt_begin + it;
         int page = 0;
         if (lane < 8) page = pt[min(kt * 8 + lane, pg_max)];
         if (lane == 0) {
@@ -224,13 +275,13 @@ attention_kernel(const __grid_constant__ AttnLaunch p, const __grid_constant__ A
           const int gp = layer * p.n_pages + page;
           const uint32_t kdst = sbase + OFF_K + st * kTileBytes + lane * 2048;
           const uint32_t vdst = sbase + OFF_V + st * kTileBytes;
-          tma_load_4d(kdst, &maps.k, bar(B_KF + st), 0, 0, t.kv, gp);
-          tma_load_4d(kdst + kHalf, &maps.k, bar(B_KF + st), 64, 0, t.kv, gp);
+          tma_load_4d(kdst, &maps.k, bar(B_KF + st), 0, 0, w.kv, gp);
+          tma_load_4d(kdst + kHalf, &maps.k, bar(B_KF + st), 64, 0, w.kv, gp);
           if (!vt) {
-            tma_load_4d(vdst + lane * 2048, &maps.v, bar(B_VF + st), 0, 0, t.kv, gp);
-            tma_load_4d(vdst + lane * 2048 + kHalf, &maps.v, bar(B_VF + st), 64, 0, t.kv, gp);
+            tma_load_4d(vdst + lane * 2048, &maps.v, bar(B_VF + st), 0, 0, w.kv, gp);
+            tma_load_4d(vdst + lane * 2048 + kHalf, &maps.v, bar(B_VF + st), 64, 0, w.kv, gp);
           } else {
-            tma_load_4d(vdst + lane * 4096, &maps.v, bar(B_VF + st), 0, 0, t.kv, gp);
+            tma_load_4d(vdst + lane * 4096, &maps.v, bar(B_VF + st), 0, 0, w.kv, gp);
           }
         }
         issued = it + 1;
@@ -248,213 +299,209 @@ attention_kernel(const __grid_constant__ AttnLaunch p, const __grid_constant__ A
     // ------------------------------------------------------ MMA issuer
     constexpr uint32_t idesc_qk = idesc_bf16_f32(BM, BN, false);
     const uint32_t idesc_pv = idesc_bf16_f32(BM, D, !vt);
+    auto issue_s = [&](int x, int st) {   // S_x = Q_x K^T
+      const uint32_t qa = sbase + OFF_Q + x * kTileBytes;
+      const uint32_t ka = sbase + OFF_K + st * kTileBytes;
+#pragma unroll
+      for (int kk = 0; kk < D / 16; ++kk) {
+        const uint32_t off = (kk >> 2) * kHalf + (kk & 3) * 32;
+        mma_bf16(tmem + TM_S + x * 128, smem_desc(qa + off, 16, 1024, kSwizzle128B),
+                 smem_desc(ka + off, 16, 1024, kSwizzle128B), idesc_qk, kk > 0);
+      }
+      mma_commit(bar(B_SF + x));
+    };
+    auto issue_pv = [&](int x, int st, bool first) {   // O_x += P_x V
+      const uint32_t va = sbase + OFF_V + st * kTileBytes;
+#pragma unroll
+      for (int kk = 0; kk < BN / 16; ++kk) {
+        // row-major V: MN-major, 64-wide d halves 16 KiB apart (LBO), 8-key
+        // groups 1 KiB apart (SBO); token-innermost V: K-major pages of
+        // [128 d][16 keys], 8-row groups 256 B apart. P: 16 keys = 8 columns.
+        const uint64_t bdesc = vt ? smem_desc(va + kk * 4096, 16, 256, kSwizzle32B)
+                                  : smem_desc(va + kk * 2048, kHalf, 1024, kSwizzle128B);
+        mma_bf16_ts(tmem + TM_O + x * 128, tmem + TM_S + x * 128 + kk * 8, bdesc, idesc_pv,
+                    (!first || kk > 0) ? 1u : 0u);
+      }
+    };
     bool ok = true;
     if (n_tiles > 0) {
-      ok = mbar_wait(bar(B_Q), 0, kBudgetNs, abort, gabort);
-      ok = __all_sync(0xffffffffu, ok);
-      for (int it = 0; ok && it <= n_tiles; ++it) {
-        if (it < n_tiles) {
-          const int st = it & 1;
-          bool w = mbar_wait(bar(B_KF + st), (it >> 1) & 1, kBudgetNs, abort, gabort);
-          if (w && it >= 2) w = mbar_wait(bar(B_SFREE + st), ((it >> 1) - 1) & 1, kBudgetNs, abort, gabort);
-          ok = __all_sync(0xffffffffu, w);
+      bool wt = mbar_wait(bar(B_Q), 0, kBudgetNs, abort, gabort);
+      if (wt) wt = mbar_wait(bar(B_KF), 0, kBudgetNs, abort, gabort);
+      ok = __all_sync(0xffffffffu, wt);
+      if (ok) {
+        tc_fence_after();
+        if (lane == 0)
+          for (int x = 0; x < n_q; ++x) issue_s(x, 0);
+        __syncwarp();
+      }
+      for (int j = 0; ok && j < n_tiles; ++j) {
+        const int st = j & 1;
+        for (int x = 0; x < n_q; ++x) {
+          wt = mbar_wait(bar(B_PF + x), j & 1, kBudgetNs, abort, gabort);
+          if (wt && x == 0) wt = mbar_wait(bar(B_VF + st), (j >> 1) & 1, kBudgetNs, abort, gabort);
+          if (wt && x == 0 && j + 1 < n_tiles)
+            wt = mbar_wait(bar(B_KF + ((j + 1) & 1)), ((j + 1) >> 1) & 1, kBudgetNs, abort, gabort);
+          ok = __all_sync(0xffffffffu, wt);
           if (!ok) break;
-          tc_fence_after();
-          if (lane == 0) {
-            const uint32_t qa = sbase + OFF_Q;
-            const uint32_t ka = sbase + OFF_K + st * kTileBytes;
-#pragma unroll
-            for (int kk = 0; kk < D / 16; ++kk) {
-              const uint32_t off = (kk >> 2) * kHalf + (kk & 3) * 32;
-              mma_bf16(tmem + TM_S0 + st * 128, smem_desc(qa + off, 16, 1024, kSwizzle128B),
-                       smem_desc(ka + off, 16, 1024, kSwizzle128B), idesc_qk, kk > 0);
+          if (x == 0) {
+            const int key0 = (w.kt_begin + j) * BN;
+            if (key0 + BN > sq.kv_len) {
+              zero_v_rows(smem + OFF_V + st * kTileBytes, sq.kv_len - key0, vt, lane);
+              fence_proxy_async_smem();
+              __syncwarp();
             }
-            mma_commit(bar(B_SF + st));
-          }
-          __syncwarp();
-        }
-        if (it >= 1) {
-          const int j = it - 1;
-          const int st = j & 1;
-          bool w = mbar_wait(bar(B_PF), j & 1, kBudgetNs, abort, gabort);
-          if (w) w = mbar_wait(bar(B_VF + st), (j >> 1) & 1, kBudgetNs, abort, gabort);
-          ok = __all_sync(0xffffffffu, w);
-          if (!ok) break;
-          const int key0 = (t.kt_begin + j) * BN;
-          if (key0 + BN > sq.kv_len) {
-            zero_v_rows(smem + OFF_V + st * kTileBytes, sq.kv_len - key0, vt, lane);
-            fence_proxy_async_smem();
-            __syncwarp();
           }
           tc_fence_after();
           if (lane == 0) {
-            const uint32_t pa = sbase + OFF_P;
-            const uint32_t va = sbase + OFF_V + st * kTileBytes;
-#pragma unroll
-            for (int kk = 0; kk < BN / 16; ++kk) {
-              const uint64_t adesc =
-                  smem_desc(pa + (kk >> 2) * kHalf + (kk & 3) * 32, 16, 1024, kSwizzle128B);
-              // row-major V: MN-major, 64-wide d halves 16 KiB apart (LBO), 8-key
-              // groups 1 KiB apart (SBO); token-innermost V: K-major pages of
-              // [128 d][16 keys], 8-row groups 256 B apart.
-              const uint64_t bdesc = vt ? smem_desc(va + kk * 4096, 16, 256, kSwizzle32B)
-                                        : smem_desc(va + kk * 2048, kHalf, 1024, kSwizzle128B);
-              mma_bf16(tmem + TM_O, adesc, bdesc, idesc_pv, (j > 0 || kk > 0) ? 1u : 0u);
-            }
-            mma_commit(bar(B_OD));
-            mma_commit(bar(B_KVE + st));
+            issue_pv(x, st, j == 0);
+            if (x == n_q - 1) mma_commit(bar(B_KVE + st));
+            if (j + 1 < n_tiles) issue_s(x, (j + 1) & 1);
+            else mma_commit(bar(B_OD + x));
           }
           __syncwarp();
         }
       }
       if (!ok && lane == 0) record_timeout(abort);
-    }
-    // Every MMA this thread issued has finished before TMEM is released.
-    if (n_tiles > 0) {
+      // Every MMA this thread issued has finished before TMEM is released.
       if (lane == 0) mma_commit(bar(B_FIN));
       __syncwarp();
       mbar_wait(bar(B_FIN), 0, kDrainNs, never);
     }
   } else {
-    // ------------------------------------------------------ softmax warps
-    const int r = threadIdx.x;                 // tile row == TMEM lane
-    const uint32_t lane_base = static_cast<uint32_t>(warp * 32) << 16;
+    // ------------------------------------------------------ softmax warpgroups
+    const int x = warp >> 2;                   // query tile of this warpgroup
+    const int r = threadIdx.x & 127;           // tile row == TMEM lane
+    const uint32_t lane_base = static_cast<uint32_t>((warp & 3) * 32) << 16;
+    const uint32_t t_s = tmem + lane_base + TM_S + x * 128;
+    const uint32_t t_o = tmem + lane_base + TM_O + x * 128;
     const int tr = r / G;                      // token within the tile
-    const int pos_r = t.pos0 + tr;
-    const bool row_valid = (r < G * p.tile_tokens) && (tr < t.ntok);
-    float m_run = -INFINITY;
+    const int pos_r = (x ? w.pos0[1] : w.pos0[0]) + tr;
+    const int ntok_x = x ? w.ntok[1] : w.ntok[0];
+    const int tok0_x = x ? w.tok0[1] : w.tok0[0];
+    const bool active = x < n_q && n_tiles > 0;
+    const bool row_valid = x < n_q && (r < G * p.tile_tokens) && (tr < ntok_x);
+    const float sc = p.scale_log2;
+    float m_run = -INFINITY;                   // running max, log2-scaled units
     float l_run = 0.f;
     bool ok = true;
-    for (int it = 0; it < n_tiles; ++it) {
-      const int sb = it & 1;
-      bool w = mbar_wait(bar(B_SF + sb), (it >> 1) & 1, kBudgetNs, abort, gabort);
-      ok = __all_sync(0xffffffffu, w);
+    for (int j = 0; active && j < n_tiles; ++j) {
+      bool wt = mbar_wait(bar(B_SF + x), j & 1, kBudgetNs, abort, gabort);
+      ok = __all_sync(0xffffffffu, wt);
       if (!ok) break;
       tc_fence_after();
       float s[BN];
+      {
+        uint32_t v[4][32];
 #pragma unroll
-      for (int q = 0; q < 4; ++q) {
-        uint32_t v[32];
-        tmem_ld32(tmem + lane_base + TM_S0 + sb * 128 + q * 32, v);
+        for (int q = 0; q < 4; ++q) tmem_ld32(t_s + q * 32, v[q]);
         tmem_ld_wait();
 #pragma unroll
-        for (int e = 0; e < 32; ++e) s[q * 32 + e] = __uint_as_float(v[e]);
-      }
-      tc_fence_before();
-      mbar_arrive(bar(B_SFREE + sb));
-
-      const int lim = pos_r - (t.kt_begin + it) * BN;   // keys j <= lim are visible
-      float mx = -INFINITY;
-      if (lim >= BN - 1) {
+        for (int q = 0; q < 4; ++q)
 #pragma unroll
-        for (int j = 0; j < BN; ++j) { s[j] *= p.scale_log2; mx = fmaxf(mx, s[j]); }
-      } else {
-#pragma unroll
-        for (int j = 0; j < BN; ++j) {
-          s[j] = (j <= lim) ? s[j] * p.scale_log2 : -INFINITY;
-          mx = fmaxf(mx, s[j]);
-        }
+          for (int e = 0; e < 32; ++e) s[q * 32 + e] = __uint_as_float(v[q][e]);
       }
+      const int lim = pos_r - (w.kt_begin + j) * BN;   // keys c <= lim are visible
+      if (lim < BN - 1) {
+#pragma unroll
+        for (int c = 0; c < BN; ++c) s[c] = (c <= lim) ? s[c] : -INFINITY;
+      }
+      float mx = fmax3(s[0], s[1], s[2]);
+#pragma unroll
+      for (int c = 3; c + 1 < BN; c += 2) mx = fmax3(mx, s[c], s[c + 1]);
+      mx = fmaxf(mx, s[BN - 1]);
+      const float mxs = mx * sc;
       // Move the running max only when the new one is far above it; the
       // stale max keeps every p <= 2^8 and O / l unchanged.
       float alpha = 1.f;
       bool rescale = false;
-      if (mx > -INFINITY && (m_run == -INFINITY || mx > m_run + kRescaleThreshold)) {
-        if (m_run != -INFINITY) { alpha = ex2_approx(m_run - mx); rescale = true; }
-        m_run = mx;
+      if (mx > -INFINITY && (m_run == -INFINITY || mxs > m_run + kRescaleThreshold)) {
+        if (m_run != -INFINITY) { alpha = ex2_approx(m_run - mxs); rescale = true; }
+        m_run = mxs;
       }
-      const float m_use = (m_run == -INFINITY) ? 0.f : m_run;
-      uint32_t pk[BN / 2];
-      float sum = 0.f;
+      const float neg_m = (m_run == -INFINITY) ? 0.f : -m_run;
+      float sum0 = 0.f, sum1 = 0.f;
 #pragma unroll
-      for (int j = 0; j < BN; j += 2) {
-        const float p0 = ex2_approx(s[j] - m_use);
-        const float p1 = ex2_approx(s[j + 1] - m_use);
-        sum += p0 + p1;
-        pk[j / 2] = pack_bf16x2(p0, p1);
+      for (int q = 0; q < 8; ++q) {
+        uint32_t pk[8];
+#pragma unroll
+        for (int e = 0; e < 16; e += 2) {
+          float a = s[q * 16 + e], b = s[q * 16 + e + 1];
+          a = ex2_approx(fmaf(a, sc, neg_m));
+          b = ex2_approx(fmaf(b, sc, neg_m));
+          sum0 += a; sum1 += b;
+          pk[e / 2] = pack_bf16x2(a, b);
+        }
+        tmem_st8(t_s + q * 8, pk);   // P over the first 64 columns of S
       }
-      l_run = l_run * alpha + sum;
-
-      if (it >= 1) {
-        // PV of the previous tile must be done before O is rescaled and P reused.
-        w = mbar_wait(bar(B_OD), (it - 1) & 1, kBudgetNs, abort, gabort);
-        ok = __all_sync(0xffffffffu, w);
-        if (!ok) break;
-        tc_fence_after();
-        if (__any_sync(0xffffffffu, rescale)) {
+      if (__any_sync(0xffffffffu, rescale)) {
+        // PV_x(j-1) is complete: this step's S-full barrier was committed after it.
+#pragma unroll 1
+        for (int q = 0; q < 4; ++q) {
+          uint32_t v[32];
+          tmem_ld32(t_o + q * 32, v);
+          tmem_ld_wait();
 #pragma unroll
-          for (int q = 0; q < 4; ++q) {
-            uint32_t v[32];
-            tmem_ld32(tmem + lane_base + TM_O + q * 32, v);
-            tmem_ld_wait();
-#pragma unroll
-            for (int e = 0; e < 32; ++e) v[e] = __float_as_uint(__uint_as_float(v[e]) * alpha);
-            tmem_st32(tmem + lane_base + TM_O + q * 32, v);
-          }
-          tmem_st_wait();
+          for (int e = 0; e < 32; ++e) v[e] = __float_as_uint(__uint_as_float(v[e]) * alpha);
+          tmem_st32(t_o + q * 32, v);
         }
       }
-      // P row -> shared memory, K-major with the 128-byte swizzle.
-      const uint32_t prow = sbase + OFF_P + r * 128;
-#pragma unroll
-      for (int c = 0; c < BN / 8; ++c) {
-        const uint32_t addr = prow + (c >> 3) * kHalf + (((c & 7) ^ (r & 7)) << 4);
-        st_shared_v4(addr, pk[c * 4], pk[c * 4 + 1], pk[c * 4 + 2], pk[c * 4 + 3]);
-      }
-      fence_proxy_async_smem();
+      tmem_st_wait();
+      l_run = l_run * alpha + (sum0 + sum1);
       tc_fence_before();
-      mbar_arrive(bar(B_PF));
+      mbar_arrive(bar(B_PF + x));
     }
     if (!ok && r == 0) record_timeout(abort);
 
-    // ---- epilogue: O / l and LSE
-    float o[D];
+    // ---- epilogue: O / l and LSE, 32 columns at a time
     bool have_o = false;
-    if (ok && n_tiles > 0) {
-      bool w = mbar_wait(bar(B_OD), (n_tiles - 1) & 1, kBudgetNs, abort, gabort);
-      w = __all_sync(0xffffffffu, w);
-      if (w) {
-        tc_fence_after();
+    if (active && ok) {
+      bool wt = mbar_wait(bar(B_OD + x), 0, kBudgetNs, abort, gabort);
+      have_o = __all_sync(0xffffffffu, wt);
+      if (!have_o && r == 0) record_timeout(abort);
+      if (have_o) tc_fence_after();
+    }
+    const bool good = have_o && l_run > 0.f;
+    const float inv_l = good ? 1.f / l_run : 0.f;
+    const float lse = good ? (m_run + log2f(l_run)) * 0.69314718055994531f : -INFINITY;
+    const int tok = sq.q_off + tok0_x + tr;
+    const int head = w.kv * G + (r % G);
+    const int64_t row = ((int64_t)w.layer_rel * p.n_tok + tok) * p.n_q_heads + head;
+    const int64_t rows_per_split = (int64_t)p.n_layers_call * p.n_tok * p.n_q_heads;
 #pragma unroll
-        for (int q = 0; q < 4; ++q) {
-          uint32_t v[32];
-          tmem_ld32(tmem + lane_base + TM_O + q * 32, v);
-          tmem_ld_wait();
+    for (int q = 0; q < 4; ++q) {
+      uint32_t v[32];
+      if (have_o) {
+        tmem_ld32(t_o + q * 32, v);
+        tmem_ld_wait();
+      }
+      if (!row_valid) continue;
+      if (p.splits == 1) {
+        uint4* dst = reinterpret_cast<uint4*>(p.out + row * D + q * 32);
 #pragma unroll
-          for (int e = 0; e < 32; ++e) o[q * 32 + e] = __uint_as_float(v[e]);
+        for (int c = 0; c < 4; ++c) {
+          float f[8];
+#pragma unroll
+          for (int e = 0; e < 8; ++e) f[e] = have_o ? __uint_as_float(v[c * 8 + e]) * inv_l : 0.f;
+          dst[c] = make_uint4(pack_bf16x2(f[0], f[1]), pack_bf16x2(f[2], f[3]),
+                              pack_bf16x2(f[4], f[5]), pack_bf16x2(f[6], f[7]));
         }
-        have_o = true;
-      } else if (r == 0) {
-        record_timeout(abort);
+      } else {
+        float4* dst = reinterpret_cast<float4*>(
+            p.part_o + ((int64_t)w.split * rows_per_split + row) * D + q * 32);
+#pragma unroll
+        for (int c = 0; c < 8; ++c)
+          dst[c] = have_o ? make_float4(__uint_as_float(v[4 * c]) * inv_l,
+                                        __uint_as_float(v[4 * c + 1]) * inv_l,
+                                        __uint_as_float(v[4 * c + 2]) * inv_l,
+                                        __uint_as_float(v[4 * c + 3]) * inv_l)
+                          : make_float4(0.f, 0.f, 0.f, 0.f);
       }
     }
     if (row_valid) {
-      const float inv_l = (have_o && l_run > 0.f) ? 1.f / l_run : 0.f;
-      const float lse = (have_o && l_run > 0.f) ? (m_run + log2f(l_run)) * 0.69314718055994531f
-                                               : -INFINITY;
-      const int tok = sq.q_off + t.tok0 + tr;
-      const int head = t.kv * G + (r % G);
-      const int64_t row = ((int64_t)t.layer_rel * p.n_tok + tok) * p.n_q_heads + head;
       if (p.splits == 1) {
-        uint4* dst = reinterpret_cast<uint4*>(p.out + row * D);
-#pragma unroll
-        for (int c = 0; c < D / 8; ++c) {
-          float v[8];
-#pragma unroll
-          for (int e = 0; e < 8; ++e) v[e] = have_o ? o[c * 8 + e] * inv_l : 0.f;
-          dst[c] = make_uint4(pack_bf16x2(v[0], v[1]), pack_bf16x2(v[2], v[3]),
-                              pack_bf16x2(v[4], v[5]), pack_bf16x2(v[6], v[7]));
-        }
         if (p.lse) p.lse[row] = lse;
       } else {
-        const int64_t rows_per_split = (int64_t)p.n_layers_call * p.n_tok * p.n_q_heads;
-        float4* dst = reinterpret_cast<float4*>(p.part_o + ((int64_t)t.split * rows_per_split + row) * D);
-#pragma unroll
-        for (int c = 0; c < D / 4; ++c)
-          dst[c] = have_o ? make_float4(o[4 * c] * inv_l, o[4 * c + 1] * inv_l,
-                                        o[4 * c + 2] * inv_l, o[4 * c + 3] * inv_l)
-                          : make_float4(0.f, 0.f, 0.f, 0.f);
-        p.part_lse[(int64_t)t.split * rows_per_split + row] = lse;
+        p.part_lse[(int64_t)w.split * rows_per_split + row] = lse;
       }
     }
   }

@@ -99,9 +99,9 @@ struct AttnLaunch {
   int32_t n_seqs;
   int32_t splits;
   int32_t v_transposed;
-  int32_t total_tiles;      // sum over sequences of q tiles
+  int32_t total_tiles;      // CTAs per (KV head, layer, split): pairs of 128-row query tiles
   float scale_log2;         // log2(e) / sqrt(head_dim)
-  int32_t tile_prefix[kMaxSeqs + 1];
+  int32_t tile_prefix[kMaxSeqs + 1];   // first CTA (tile pair) of each sequence
   AttnSeq seq[kMaxSeqs];
 };
 

@@ -255,7 +255,7 @@ nexus_status plan_attention(int32_t n_seqs, const int32_t* kv_len, const int32_t
   for (int32_t s = 0; s < n_seqs; ++s) {
     if (q_len[s] < 0 || kv_len[s] < q_len[s]) return NEXUS_EINVAL;
     tok += q_len[s];
-    tiles += (q_len[s] + tile_tokens - 1) / tile_tokens;
+    tiles += ((q_len[s] + tile_tokens - 1) / tile_tokens + 1) / 2;   // CTAs: pairs of query tiles
     if (q_len[s] > 0) pl.kt_max = std::max(pl.kt_max, (kv_len[s] + 127) / 128);
   }
   if (tok > 0x7FFFFFFF || tiles > 0x7FFFFFFF) return NEXUS_ERANGE;
@@ -268,7 +268,9 @@ nexus_status plan_attention(int32_t n_seqs, const int32_t* kv_len, const int32_t
     const int sms = num_sms();
     int best = 1;
     double best_cost = 1e300;
-    if (ctas > 0 && pl.kt_max > 0) {
+    // Splitting the keys only pays when the query tiles alone fill less than
+    // one wave of the GPU (short suffixes over deep caches).
+    if (ctas > 0 && ctas < sms && pl.kt_max > 0) {
       for (int s = 1; s <= std::min<int>(kMaxSplits, pl.kt_max); ++s) {
         const double waves = std::ceil(static_cast<double>(ctas) * s / sms);
         const double cost = waves * std::ceil(static_cast<double>(pl.kt_max) / s) + (s > 1 ? 2.0 : 0.0);
@@ -346,7 +348,7 @@ nexus_status attention_impl(const nexus_kv_cache* c, const int32_t* d_pt, int32_
     p->seq[s].q_len = q_len[s];
     p->seq[s].q_off = off;
     p->seq[s].pt_row = h_rows ? h_rows[s] : s;
-    tiles += (q_len[s] + p->tile_tokens - 1) / p->tile_tokens;
+    tiles += ((q_len[s] + p->tile_tokens - 1) / p->tile_tokens + 1) / 2;
     off += q_len[s];
   }
   p->tile_prefix[n_seqs] = tiles;
