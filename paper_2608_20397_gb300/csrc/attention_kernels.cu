@@ -11,10 +11,10 @@
 //              (eight 16-token pages each, through the page table) into a
 //              two-stage ring
 //   warp 9     MMA issuer (tcgen05.mma, bf16 in, f32 accumulate in TMEM):
-//              S_A(0) S_B(0), then per key tile j:
-//              PV_A(j) S_A(j+1) PV_B(j) S_B(j+1)
-//              so the tensor core always has two products queued while one
-//              softmax warpgroup works
+//              S_A(0) S_B(0), then batches PV_A(j) S_A(j+1) | PV_B(j) S_B(j+1),
+//              in this order, so one tile's products run while the other
+//              tile's softmax works. The barriers a batch needs are waited on
+//              by different lanes at once.
 //   warps 0-3  softmax of tile A, warps 4-7 softmax of tile B: thread i of a
 //              warpgroup owns TMEM lane i (= tile row i); online softmax in the
 //              log2 domain, the running max moved only past 2^8 growth (then O
@@ -59,14 +59,16 @@ constexpr uint32_t OFF_V = OFF_K + kStages * kTileBytes;
 constexpr uint32_t OFF_BAR = OFF_V + kStages * kTileBytes;
 enum {
   B_Q = 0,
-  B_KF = 1,      // +stage
-  B_VF = 3,      // +stage
-  B_KVE = 5,     // +stage
-  B_SF = 7,      // +tile
-  B_PF = 9,      // +tile
-  B_OD = 11,     // +tile
-  B_FIN = 13,
-  kNumBars = 14
+  B_KF = 1,      // +stage: K tile landed
+  B_VF = 3,      // +stage: V tile landed
+  B_KE = 5,      // +stage: K tile consumed (every tile's S product done)
+  B_VE = 7,      // +stage: V tile consumed (every tile's P V product done)
+  B_SF = 9,      // +tile
+  B_PF = 11,     // +tile
+  B_OD = 13,     // +tile
+  B_FIN = 15,
+  B_VZ = 16,     // last V tile's rows past kv_len are zeroed
+  kNumBars = 17
 };
 constexpr uint32_t OFF_MISC = OFF_BAR + kNumBars * 8;
 constexpr uint32_t kSmemUsed = OFF_MISC + 16;
@@ -149,6 +151,28 @@ __device__ __forceinline__ float fmax3(float a, float b, float c) {
   return d;
 }
 
+// 2^x on the FMA pipe, to take part of the exponentials off the MUFU unit:
+// 2^x = 2^n * 2^f with n = rint(x) (by the 1.5 * 2^23 rounding constant) and
+// f = x - n in [-0.5, 0.5]; 2^f is a degree-3 polynomial fitted here for the
+// least maximum relative error on that interval (7.5e-5, far below the bf16
+// resolution of P); n is added into the exponent field. Below 2^-125 the
+// result is exactly 0, so masked scores (-inf) still give p = 0.
+constexpr float kExp2C0 = 0.99992806f;
+constexpr float kExp2C1 = 0.69326097f;
+constexpr float kExp2C2 = 0.24261113f;
+constexpr float kExp2C3 = 0.05517167f;
+constexpr int kPolyPairsPer8 = 0;   // pairs (of every 8) whose exponentials use the polynomial
+
+__device__ __forceinline__ float exp2_poly(float x) {
+  const float xc = fmaxf(x, -125.f);
+  const float t = __fadd_rn(xc, 12582912.f);
+  const float n = __fsub_rn(t, 12582912.f);
+  const float f = __fsub_rn(xc, n);
+  const float p = fmaf(fmaf(fmaf(kExp2C3, f, kExp2C2), f, kExp2C1), f, kExp2C0);
+  const float y = __int_as_float(__float_as_int(p) + (__float_as_int(t) << 23));
+  return x < -125.f ? 0.f : y;
+}
+
 // D[tmem] (+)= A[tmem] * B[smem]: A is read from tensor memory (P, packed
 // bf16 pairs along K, row i in lane i).
 __device__ __forceinline__ void mma_bf16_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t b_desc,
@@ -218,7 +242,8 @@ attention_kernel(const __grid_constant__ AttnLaunch p, const __grid_constant__ A
     for (int s = 0; s < kStages; ++s) {
       mbar_init(bar(B_KF + s), 1);
       mbar_init(bar(B_VF + s), 1);
-      mbar_init(bar(B_KVE + s), 1);
+      mbar_init(bar(B_KE + s), 1);
+      mbar_init(bar(B_VE + s), 1);
     }
     for (int x = 0; x < 2; ++x) {
       mbar_init(bar(B_SF + x), 1);
@@ -226,6 +251,7 @@ attention_kernel(const __grid_constant__ AttnLaunch p, const __grid_constant__ A
       mbar_init(bar(B_OD + x), 1);
     }
     mbar_init(bar(B_FIN), 1);
+    mbar_init(bar(B_VZ), 1);
     *abort = 0;
     *never = 0;
     fence_mbar_init();
@@ -244,7 +270,7 @@ attention_kernel(const __grid_constant__ AttnLaunch p, const __grid_constant__ A
     // ------------------------------------------------------ TMA producer
     const int32_t* pt = p.page_tables + (int64_t)sq.pt_row * p.max_pages;
     const int pg_max = (sq.kv_len - 1) / kPageSize;
-    int issued = 0;
+    int issued = 0, issued_k = 0;
     if (n_tiles > 0) {
       if (lane == 0) {
         prefetch_tmap(&maps.q);
@@ -256,27 +282,33 @@ attention_kernel(const __grid_constant__ AttnLaunch p, const __grid_constant__ A
             tma_load_4d(sbase + OFF_Q + x * kTileBytes + half * kHalf, &maps.q, bar(B_Q),
                         half * 64, w.kv * G, sq.q_off + (x ? w.tok0[1] : w.tok0[0]), w.layer_rel);
       }
+      // K and V stages are released separately: K_j is free once both S
+      // products of tile j are done, an iteration before V_j, so K tiles are
+      // fetched a full iteration ahead of their use.
       for (int it = 0; it < n_tiles; ++it) {
         const int st = it & 1;
-        if (it >= 2) {
-          bool ok = mbar_wait(bar(B_KVE + st), ((it >> 1) - 1) & 1, kBudgetNs, abort, gabort);
-          ok = __all_sync(0xffffffffu, ok);
-          if (!ok) { if (lane == 0) record_timeout(abort); break; }
-        }
         const int kt = w.kt_begin + it;
         int page = 0;
         if (lane < 8) page = pt[min(kt * 8 + lane, pg_max)];
-        if (lane == 0) {
-          mbar_arrive_expect_tx(bar(B_KF + st), kTileBytes);
-          mbar_arrive_expect_tx(bar(B_VF + st), kTileBytes);
-        }
+        const int gp = layer * p.n_pages + page;
+        bool ok = true;
+        if (it >= 2) ok = mbar_wait(bar(B_KE + st), ((it >> 1) - 1) & 1, kBudgetNs, abort, gabort);
+        ok = __all_sync(0xffffffffu, ok);
+        if (!ok) { if (lane == 0) record_timeout(abort); break; }
+        if (lane == 0) mbar_arrive_expect_tx(bar(B_KF + st), kTileBytes);
         __syncwarp();
         if (lane < 8) {
-          const int gp = layer * p.n_pages + page;
           const uint32_t kdst = sbase + OFF_K + st * kTileBytes + lane * 2048;
-          const uint32_t vdst = sbase + OFF_V + st * kTileBytes;
           tma_load_4d(kdst, &maps.k, bar(B_KF + st), 0, 0, w.kv, gp);
           tma_load_4d(kdst + kHalf, &maps.k, bar(B_KF + st), 64, 0, w.kv, gp);
+        }
+        if (it >= 2) ok = mbar_wait(bar(B_VE + st), ((it >> 1) - 1) & 1, kBudgetNs, abort, gabort);
+        ok = __all_sync(0xffffffffu, ok);
+        if (!ok) { if (lane == 0) record_timeout(abort); issued_k = it + 1; break; }
+        if (lane == 0) mbar_arrive_expect_tx(bar(B_VF + st), kTileBytes);
+        __syncwarp();
+        if (lane < 8) {
+          const uint32_t vdst = sbase + OFF_V + st * kTileBytes;
           if (!vt) {
             tma_load_4d(vdst + lane * 2048, &maps.v, bar(B_VF + st), 0, 0, w.kv, gp);
             tma_load_4d(vdst + lane * 2048 + kHalf, &maps.v, bar(B_VF + st), 64, 0, w.kv, gp);
@@ -285,14 +317,26 @@ attention_kernel(const __grid_constant__ AttnLaunch p, const __grid_constant__ A
           }
         }
         issued = it + 1;
+        issued_k = it + 1;
+        const int key0 = kt * BN;
+        if (key0 + BN > sq.kv_len) {
+          // The tile holding the last key: cache slots past kv_len may hold any
+          // bits, so their V rows are zeroed before any P V product reads them.
+          ok = mbar_wait(bar(B_VF + st), (it >> 1) & 1, kBudgetNs, abort, gabort);
+          ok = __all_sync(0xffffffffu, ok);
+          if (!ok) { if (lane == 0) record_timeout(abort); break; }
+          zero_v_rows(smem + OFF_V + st * kTileBytes, sq.kv_len - key0, vt, lane);
+          fence_proxy_async_smem();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(bar(B_VZ));
+        }
       }
       if (*abort) {
         // Let the copies still in flight land before the CTA exits.
-        for (int it = max(0, issued - 2); it < issued; ++it) {
-          const int st = it & 1;
-          mbar_wait(bar(B_KF + st), (it >> 1) & 1, kDrainNs, never);
-          mbar_wait(bar(B_VF + st), (it >> 1) & 1, kDrainNs, never);
-        }
+        for (int it = max(0, issued_k - 2); it < issued_k; ++it)
+          mbar_wait(bar(B_KF + (it & 1)), (it >> 1) & 1, kDrainNs, never);
+        for (int it = max(0, issued - 2); it < issued; ++it)
+          mbar_wait(bar(B_VF + (it & 1)), (it >> 1) & 1, kDrainNs, never);
       }
     }
   } else if (warp == kMmaWarp) {
@@ -302,16 +346,19 @@ attention_kernel(const __grid_constant__ AttnLaunch p, const __grid_constant__ A
     auto issue_s = [&](int x, int st) {   // S_x = Q_x K^T
       const uint32_t qa = sbase + OFF_Q + x * kTileBytes;
       const uint32_t ka = sbase + OFF_K + st * kTileBytes;
+      const uint32_t t_s = tmem + TM_S + x * 128;
 #pragma unroll
       for (int kk = 0; kk < D / 16; ++kk) {
         const uint32_t off = (kk >> 2) * kHalf + (kk & 3) * 32;
-        mma_bf16(tmem + TM_S + x * 128, smem_desc(qa + off, 16, 1024, kSwizzle128B),
+        mma_bf16(t_s, smem_desc(qa + off, 16, 1024, kSwizzle128B),
                  smem_desc(ka + off, 16, 1024, kSwizzle128B), idesc_qk, kk > 0);
       }
       mma_commit(bar(B_SF + x));
     };
     auto issue_pv = [&](int x, int st, bool first) {   // O_x += P_x V
       const uint32_t va = sbase + OFF_V + st * kTileBytes;
+      const uint32_t t_s = tmem + TM_S + x * 128;
+      const uint32_t t_o = tmem + TM_O + x * 128;
 #pragma unroll
       for (int kk = 0; kk < BN / 16; ++kk) {
         // row-major V: MN-major, 64-wide d halves 16 KiB apart (LBO), 8-key
@@ -319,44 +366,52 @@ attention_kernel(const __grid_constant__ AttnLaunch p, const __grid_constant__ A
         // [128 d][16 keys], 8-row groups 256 B apart. P: 16 keys = 8 columns.
         const uint64_t bdesc = vt ? smem_desc(va + kk * 4096, 16, 256, kSwizzle32B)
                                   : smem_desc(va + kk * 2048, kHalf, 1024, kSwizzle128B);
-        mma_bf16_ts(tmem + TM_O + x * 128, tmem + TM_S + x * 128 + kk * 8, bdesc, idesc_pv,
-                    (!first || kk > 0) ? 1u : 0u);
+        mma_bf16_ts(t_o, t_s + kk * 8, bdesc, idesc_pv, (!first || kk > 0) ? 1u : 0u);
       }
+    };
+    // Lanes 0-3 wait on different barriers at once (0 = none).
+    auto wait4 = [&](uint32_t b0, uint32_t p0, uint32_t b1, uint32_t p1, uint32_t b2, uint32_t p2,
+                     uint32_t b3, uint32_t p3) -> bool {
+      uint32_t br = 0, par = 0;
+      if (lane == 0) { br = b0; par = p0; }
+      if (lane == 1) { br = b1; par = p1; }
+      if (lane == 2) { br = b2; par = p2; }
+      if (lane == 3) { br = b3; par = p3; }
+      const bool wt = br ? mbar_wait(br, par, kBudgetNs, abort, gabort) : true;
+      __syncwarp();
+      return __all_sync(0xffffffffu, wt);
     };
     bool ok = true;
     if (n_tiles > 0) {
-      bool wt = mbar_wait(bar(B_Q), 0, kBudgetNs, abort, gabort);
-      if (wt) wt = mbar_wait(bar(B_KF), 0, kBudgetNs, abort, gabort);
-      ok = __all_sync(0xffffffffu, wt);
-      if (ok) {
+      ok = wait4(bar(B_Q), 0, bar(B_KF), 0, 0, 0, 0, 0);
+      if (ok && lane == 0) {
         tc_fence_after();
-        if (lane == 0)
-          for (int x = 0; x < n_q; ++x) issue_s(x, 0);
-        __syncwarp();
+        for (int x = 0; x < n_q; ++x) issue_s(x, 0);
+        mma_commit(bar(B_KE + 0));
       }
+      __syncwarp();
       for (int j = 0; ok && j < n_tiles; ++j) {
         const int st = j & 1;
-        for (int x = 0; x < n_q; ++x) {
-          wt = mbar_wait(bar(B_PF + x), j & 1, kBudgetNs, abort, gabort);
-          if (wt && x == 0) wt = mbar_wait(bar(B_VF + st), (j >> 1) & 1, kBudgetNs, abort, gabort);
-          if (wt && x == 0 && j + 1 < n_tiles)
-            wt = mbar_wait(bar(B_KF + ((j + 1) & 1)), ((j + 1) >> 1) & 1, kBudgetNs, abort, gabort);
-          ok = __all_sync(0xffffffffu, wt);
+        const int nst = (j + 1) & 1;
+        const bool more = j + 1 < n_tiles;
+        const bool ragged = (w.kt_begin + j) * BN + BN > sq.kv_len;
+        for (int x = 0; ok && x < n_q; ++x) {
+          if (x == 0)
+            ok = wait4(bar(B_PF), j & 1, bar(B_VF + st), (j >> 1) & 1,
+                       more ? bar(B_KF + nst) : 0u, ((j + 1) >> 1) & 1, ragged ? bar(B_VZ) : 0u, 0);
+          else
+            ok = wait4(bar(B_PF + x), j & 1, 0, 0, 0, 0, 0, 0);
           if (!ok) break;
-          if (x == 0) {
-            const int key0 = (w.kt_begin + j) * BN;
-            if (key0 + BN > sq.kv_len) {
-              zero_v_rows(smem + OFF_V + st * kTileBytes, sq.kv_len - key0, vt, lane);
-              fence_proxy_async_smem();
-              __syncwarp();
-            }
-          }
-          tc_fence_after();
           if (lane == 0) {
+            tc_fence_after();
             issue_pv(x, st, j == 0);
-            if (x == n_q - 1) mma_commit(bar(B_KVE + st));
-            if (j + 1 < n_tiles) issue_s(x, (j + 1) & 1);
-            else mma_commit(bar(B_OD + x));
+            if (x == n_q - 1) mma_commit(bar(B_VE + st));
+            if (more) {
+              issue_s(x, nst);
+              if (x == n_q - 1) mma_commit(bar(B_KE + nst));
+            } else {
+              mma_commit(bar(B_OD + x));
+            }
           }
           __syncwarp();
         }
@@ -405,10 +460,18 @@ attention_kernel(const __grid_constant__ AttnLaunch p, const __grid_constant__ A
 #pragma unroll
         for (int c = 0; c < BN; ++c) s[c] = (c <= lim) ? s[c] : -INFINITY;
       }
-      float mx = fmax3(s[0], s[1], s[2]);
+      // Row max as eight independent 3-input chains, then a short tree.
+      float mxa[8];
 #pragma unroll
-      for (int c = 3; c + 1 < BN; c += 2) mx = fmax3(mx, s[c], s[c + 1]);
-      mx = fmaxf(mx, s[BN - 1]);
+      for (int k = 0; k < 8; ++k) mxa[k] = fmax3(s[k], s[8 + k], s[16 + k]);
+#pragma unroll
+      for (int c = 24; c + 16 <= BN; c += 16)
+#pragma unroll
+        for (int k = 0; k < 8; ++k) mxa[k] = fmax3(mxa[k], s[c + k], s[c + 8 + k]);
+#pragma unroll
+      for (int k = 0; k < 8; ++k) mxa[k] = fmaxf(mxa[k], s[BN - 8 + k]);
+      const float mx = fmaxf(fmax3(mxa[0], mxa[1], mxa[2]),
+                             fmaxf(fmax3(mxa[3], mxa[4], mxa[5]), fmaxf(mxa[6], mxa[7])));
       const float mxs = mx * sc;
       // Move the running max only when the new one is far above it; the
       // stale max keeps every p <= 2^8 and O / l unchanged.
@@ -419,16 +482,21 @@ attention_kernel(const __grid_constant__ AttnLaunch p, const __grid_constant__ A
         m_run = mxs;
       }
       const float neg_m = (m_run == -INFINITY) ? 0.f : -m_run;
-      float sum0 = 0.f, sum1 = 0.f;
+      float sum[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};   // eight short chains
 #pragma unroll
       for (int q = 0; q < 8; ++q) {
         uint32_t pk[8];
 #pragma unroll
         for (int e = 0; e < 16; e += 2) {
-          float a = s[q * 16 + e], b = s[q * 16 + e + 1];
-          a = ex2_approx(fmaf(a, sc, neg_m));
-          b = ex2_approx(fmaf(b, sc, neg_m));
-          sum0 += a; sum1 += b;
+          float a = fmaf(s[q * 16 + e], sc, neg_m), b = fmaf(s[q * 16 + e + 1], sc, neg_m);
+          if (((e >> 1) & 7) >= 8 - kPolyPairsPer8) {
+            a = exp2_poly(a);
+            b = exp2_poly(b);
+          } else {
+            a = ex2_approx(a);
+            b = ex2_approx(b);
+          }
+          sum[(e >> 1) & 7] += a + b;
           pk[e / 2] = pack_bf16x2(a, b);
         }
         tmem_st8(t_s + q * 8, pk);   // P over the first 64 columns of S
@@ -446,7 +514,8 @@ attention_kernel(const __grid_constant__ AttnLaunch p, const __grid_constant__ A
         }
       }
       tmem_st_wait();
-      l_run = l_run * alpha + (sum0 + sum1);
+      l_run = l_run * alpha + (((sum[0] + sum[1]) + (sum[2] + sum[3])) +
+                               ((sum[4] + sum[5]) + (sum[6] + sum[7])));
       tc_fence_before();
       mbar_arrive(bar(B_PF + x));
     }
