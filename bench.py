@@ -45,6 +45,14 @@ def attn_flops(T: int, R: int, n_layers: int) -> float:
     return 4.0 * D * HQ * (R * (T - R) + R * (R + 1) / 2.0) * n_layers
 
 
+def c5_config(L, n_past, Lb, depth, T, R, splits, world):
+    return {"workload": f"c5 deep-context: {L} layers, n_past {n_past}, {Lb}-token block at "
+                        f"{depth} (T={T}); re-prefill {n_past}x{n_past} causal + {R}-query "
+                        f"split-KV suffix, 40/8 heads, d=128",
+            "parallelism": f"replicas x{world}",
+            "l2": "inputs exceed L2 (>30 GB touched per step); no flush"}
+
+
 def max_over_ranks(x: float, dist, device) -> float:
     """Largest value of x over all ranks (identity without a process group)."""
     if dist is None:
@@ -267,7 +275,7 @@ def run_reference(args):
             "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": 1e3 * statistics.median(times), "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-            "config": {"workload": "c5 deep-context (bounded oracle sample per step)"},
+            "config": c5_config(48, 32768, 2048, 30000, 34816, 64, None, 1),
             "cpu_baseline": {"value": value, "unit": "TFLOP/s", "cores": cpu_cores(),
                              "kind": "oracle", "sample": desc},
             "e2e": {"value": value, "unit": "TFLOP/s", "h2d_bytes_per_step": 0,
@@ -389,12 +397,9 @@ def main():
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_per_step,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
             "data": "synthetic",
-            "config": {"workload": f"c5 deep-context: {wl.L} layers, n_past {wl.n_past}, "
-                                   f"{wl.Lb}-token block at {wl.depth} (T={wl.T}); re-prefill "
-                                   f"{wl.n_past}x{wl.n_past} causal + {wl.R_split}-query "
-                                   f"split-KV suffix ({wl.splits} splits), 40/8 heads, d=128",
-                       "parallelism": f"replicas x{world}",
-                       "l2": "inputs exceed L2 (>30 GB touched per step); no flush"},
+            "config": c5_config(wl.L, wl.n_past, wl.Lb, wl.depth, wl.T, wl.R_split, wl.splits,
+                                world),
+            "suffix_splits": wl.splits,
             "splice_gbs": splice_gbs, "splice_ms": splice_ms, "reprefill_ms": pre_ms,
             "suffix_ms": suf_ms, "suffix_tflops": suf_tflops,
             "roofline": roofline, "roofline_splice": roofline_splice,
@@ -463,44 +468,76 @@ def _profiled_traffic(kernel: str):
 
 def _e2e(wl, stream, args, barrier, world, dist, dev):
     """The same step through the C ABI with host buffers: every step copies the
-    block K/V and every layer's Q from pinned host memory and reads every
-    layer's O back, inside the timed region."""
+    block K/V and every layer's Q in from pinned host memory and reads every
+    layer's O back, inside the timed region. Copies run on their own streams,
+    double-buffered per layer, so they overlap the attention of other layers."""
     import torch
     L = wl.L
+    nexus = wl.nexus
     h_bk = torch.empty(wl.bk.shape, dtype=torch.bfloat16, pin_memory=True)
     h_bv = torch.empty(wl.bv.shape, dtype=torch.bfloat16, pin_memory=True)
     h_bk.copy_(wl.bk)
     h_bv.copy_(wl.bv)
-    h_q = torch.empty(wl.q_pre.shape[1:], dtype=torch.bfloat16, pin_memory=True)
-    h_o = torch.empty(wl.o_pre.shape[1:], dtype=torch.bfloat16, pin_memory=True)
+    h_q = torch.empty(wl.q_pre.shape, dtype=torch.bfloat16, pin_memory=True)   # every layer's Q
+    h_o = torch.empty((2,) + tuple(wl.o_pre.shape[1:]), dtype=torch.bfloat16, pin_memory=True)
     h_qs = torch.empty(wl.q_suf.shape, dtype=torch.bfloat16, pin_memory=True)
     h_os = torch.empty(wl.o_suf.shape, dtype=torch.bfloat16, pin_memory=True)
-    h_q.copy_(wl.q_pre[0])
+    h_q.copy_(wl.q_pre)
     h_qs.copy_(wl.q_suf)
-    qbuf = torch.empty_like(wl.q_pre[:1])
-    obuf = torch.empty_like(wl.o_pre[:1])
-    h2d = (h_bk.numel() + h_bv.numel() + L * h_q.numel() + h_qs.numel()) * 2
-    d2h = (L * h_o.numel() + h_os.numel()) * 2
+    qbuf = [torch.empty_like(wl.q_pre[:1]) for _ in range(2)]
+    obuf = [torch.empty_like(wl.o_pre[:1]) for _ in range(2)]
+    s_in = torch.cuda.Stream(device=dev)
+    s_out = torch.cuda.Stream(device=dev)
+    h2d = (h_bk.numel() + h_bv.numel() + h_q.numel() + h_qs.numel()) * 2
+    d2h = (L * h_o[0].numel() + h_os.numel()) * 2
+    ev = lambda: torch.cuda.Event()
 
     def one():
-        wl.bk.copy_(h_bk, non_blocking=True)
-        wl.bv.copy_(h_bv, non_blocking=True)
-        wl.q_suf.copy_(h_qs, non_blocking=True)
-
-        nexus = wl.nexus
+        e_blk = ev()
+        with torch.cuda.stream(s_in):
+            wl.bk.copy_(h_bk, non_blocking=True)
+            wl.bv.copy_(h_bv, non_blocking=True)
+            wl.q_suf.copy_(h_qs, non_blocking=True)
+            e_blk.record(s_in)
+        stream.wait_event(e_blk)
         nexus.splice_kv(wl.cache, wl.d_pt, wl.h_pt, 2, wl.max_pages, wl.blocks, wl.segs, 0, L,
                         stream)
+        e_in = [None] * L
+        e_done = [None] * L
+        e_out = [None] * L
         for l in range(L):
-            qbuf[0].copy_(h_q, non_blocking=True)
-            nexus.reprefill(wl.cache, wl.d_pt, 2, wl.max_pages, [wl.n_past], qbuf, obuf,
-                            wl.lse_pre[l:l + 1], HQ, l, l + 1, rows=[0], split_kv=1, stream=stream)
-            h_o.copy_(obuf[0], non_blocking=True)
+            b = l & 1
+            with torch.cuda.stream(s_in):
+                if l >= 2:
+                    s_in.wait_event(e_done[l - 2])     # attention of layer l-2 read qbuf[b]
+                qbuf[b][0].copy_(h_q[l], non_blocking=True)
+                e_in[l] = ev()
+                e_in[l].record(s_in)
+            stream.wait_event(e_in[l])
+            if l >= 2:
+                stream.wait_event(e_out[l - 2])        # O of layer l-2 left obuf[b]
+            nexus.reprefill(wl.cache, wl.d_pt, 2, wl.max_pages, [wl.n_past], qbuf[b], obuf[b],
+                            wl.lse_pre[l:l + 1], HQ, l, l + 1, rows=[0], split_kv=1,
+                            stream=stream)
+            e_done[l] = ev()
+            e_done[l].record(stream)
+            with torch.cuda.stream(s_out):
+                s_out.wait_event(e_done[l])
+                h_o[b].copy_(obuf[b][0], non_blocking=True)
+                e_out[l] = ev()
+                e_out[l].record(s_out)
         for l in range(L):
             nexus.suffix_attention(wl.cache, wl.d_pt, 2, wl.max_pages, [wl.T], [wl.R_split],
                                    wl.q_suf[l:l + 1], wl.o_suf[l:l + 1], wl.lse_suf[l:l + 1], HQ,
                                    l, l + 1, rows=[1], split_kv=0, workspace=wl.ws,
                                    workspace_bytes=wl.ws_bytes, stream=stream)
-        h_os.copy_(wl.o_suf, non_blocking=True)
+        e_suf = ev()
+        e_suf.record(stream)
+        with torch.cuda.stream(s_out):
+            s_out.wait_event(e_suf)
+            h_os.copy_(wl.o_suf, non_blocking=True)
+        stream.wait_stream(s_out)
+        stream.wait_stream(s_in)
 
     for _ in range(max(1, min(args.warmup, 2))):
         one()
@@ -513,8 +550,8 @@ def _e2e(wl, stream, args, barrier, world, dist, dev):
     per = secs / args.steps
     flops = wl.flops_pre + wl.flops_suf
     return {"value": job_throughput(flops, world, per * 1e3), "unit": "TFLOP/s",
-            "ms_per_step": per * 1e3,
-            "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h)}
+            "ms_per_step": per * 1e3, "h2d_bytes_per_step": int(h2d),
+            "d2h_bytes_per_step": int(d2h)}
 
 
 if __name__ == "__main__":

@@ -90,7 +90,7 @@ class SplicedCase:
     through the C ABI. Rows 2s / 2s+1 of the page-table array are session s's
     pre- and post-splice tables."""
 
-    def __init__(self, w, dev, layers=None, spare_pages=64, garbage_fill=None):
+    def __init__(self, w, dev, layers=None, spare_pages=64, garbage_fill=None, keep_live=True):
         from paper_2608_20397_gb300.workloads import page_order
         self.w = w
         self.dev = dev
@@ -118,8 +118,10 @@ class SplicedCase:
             lk = randn_bf16((L, s.n_past, H, 128), seed + 1, dev)
             lv = randn_bf16((L, s.n_past, H, 128), seed + 2, dev)
             write_rows(self.kp, self.vp, self.h_pt[2 * si], lk, lv, self.vt)
-            self.live_k.append(lk)
-            self.live_v.append(lv)
+            # large cases regenerate the live rows from their seeds when checked
+            self.live_k.append(lk if keep_live else (L, s.n_past, H, seed + 1))
+            self.live_v.append(lv if keep_live else (L, s.n_past, H, seed + 2))
+            del lk, lv
             bks, bvs = [], []
             for j, ins in enumerate(s.inserts):
                 bk = randn_bf16((L, ins.length, H, 128), seed + 10 + 2 * j, dev)
@@ -147,6 +149,15 @@ class SplicedCase:
     def splice(self, stream=None, validate=True):
         nexus.splice_kv(self.cache, self.d_pt, self.h_pt if validate else None, self.n_rows,
                         self.max_pages, self.blocks, self.segments, 0, self.L, stream)
+
+    def live(self, si):
+        """Session si's pre-splice K and V (regenerated from the seeds if not kept)."""
+        def get(x):
+            if isinstance(x, tuple):
+                L, n, H, sd = x
+                return randn_bf16((L, n, H, 128), sd, self.dev)
+            return x
+        return get(self.live_k[si]), get(self.live_v[si])
 
     def inserts_f64(self, si, layers):
         s = self.w.sessions[si]

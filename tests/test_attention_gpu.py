@@ -147,9 +147,9 @@ def _e2e_session(case, si, R, layers, Hq=40, split_kv=1, sample_rows=None, seed=
                                rows=[2 * si + 1], split_kv=split_kv, workspace=ws,
                                workspace_bytes=nbytes)
     assert nexus.device_status() == nexus.OK
+    live_k, live_v = case.live(si)
     for li, layer in enumerate(layers):
-        want_k, want_v = oracle.splice_sequence(f64(case.live_k[si][[layer]]),
-                                                f64(case.live_v[si][[layer]]),
+        want_k, want_v = oracle.splice_sequence(f64(live_k[[layer]]), f64(live_v[[layer]]),
                                                 case.inserts_f64(si, [layer]), w.rope_theta)
         rows = np.arange(R) if sample_rows is None else sample_rows
         pos = oracle.suffix_positions(T, R)[rows]
@@ -204,6 +204,42 @@ def test_c5_reprefill_full_size_sampled_rows():
     rows = np.sort(np.concatenate([[0, 1, 24, 25, 127, 128, T - 1],
                                    rng.choice(T, size=57, replace=False)]))
     kmax = int(rows.max()) + 1
-    want_o, want_l = oracle.attention(f64(q[0, rows]), f64(case.live_k[0][layer, :kmax]),
-                                      f64(case.live_v[0][layer, :kmax]), rows, 5)
+    live_k, live_v = case.live(0)
+    want_o, want_l = oracle.attention(f64(q[0, rows]), f64(live_k[layer, :kmax]),
+                                      f64(live_v[layer, :kmax]), rows, 5)
     assert_attn_close(f64(o[0, rows]), want_o, f64(lse[0, rows]), want_l, "c5 reprefill")
+
+
+def test_end_to_end_c4_varlen_full_size():
+    """c4: 32 sessions x 48 layers spliced in one launch, then one varlen suffix
+    attention call per sampled layer over all 32 sessions (50 % of each session's
+    spliced span re-decoded), checked on sampled rows of sampled sessions."""
+    w = workload("c4")
+    case = SplicedCase(w, DEV, keep_live=False)
+    case.splice()
+    assert nexus.device_status() == nexus.OK
+    kv = [w.spliced_len(s) for s in w.sessions]
+    ql = [nexus.suffix_len(s.suffix_span, s.suffix_pct) for s in w.sessions]
+    assert ql == [oracle.redecode_len(s.suffix_span, 0, 256, s.suffix_pct, 4) for s in w.sessions]
+    rows = [2 * i + 1 for i in range(len(w.sessions))]
+    offs = np.concatenate([[0], np.cumsum(ql)])
+    rng = np.random.default_rng(44)
+    for layer in (0, 47):
+        q = randn_bf16((1, int(offs[-1]), 40, 128), 4400 + layer, DEV)
+        o = torch.empty_like(q)
+        lse = torch.empty(q.shape[:3], dtype=torch.float32, device=DEV)
+        nexus.suffix_attention(case.cache, case.d_pt, case.n_rows, case.max_pages, kv, ql, q, o,
+                               lse, 40, layer, layer + 1, rows=rows, split_kv=0)
+        assert nexus.device_status() == nexus.OK
+        for si in (0, 5, 19, 31):
+            live_k, live_v = case.live(si)
+            want_k, want_v = oracle.splice_sequence(f64(live_k[[layer]]), f64(live_v[[layer]]),
+                                                    case.inserts_f64(si, [layer]), w.rope_theta)
+            del live_k, live_v
+            sel = np.sort(rng.choice(ql[si], size=min(12, ql[si]), replace=False))
+            pos = oracle.suffix_positions(kv[si], ql[si])[sel]
+            kmax = int(pos.max()) + 1
+            want_o, want_l = oracle.attention(f64(q[0, offs[si] + sel]), want_k[0, :kmax],
+                                              want_v[0, :kmax], pos, 5)
+            assert_attn_close(f64(o[0, offs[si] + sel]), want_o, f64(lse[0, offs[si] + sel]),
+                              want_l, f"c4 session {si} layer {layer}")

@@ -20,9 +20,10 @@ def _check_session(case, si, layers):
     s = w.sessions[si]
     T = w.spliced_len(s)
     got_k, got_v = gather_rows(case.kp, case.vp, case.h_pt[2 * si + 1], T, case.vt, layers)
-    want_k, want_v = oracle.splice_sequence(f64(case.live_k[si][layers]),
-                                            f64(case.live_v[si][layers]),
+    live_k, live_v = case.live(si)
+    want_k, want_v = oracle.splice_sequence(f64(live_k[layers]), f64(live_v[layers]),
                                             case.inserts_f64(si, layers), w.rope_theta)
+    del live_k, live_v
     gk, gv = f64(got_k), f64(got_v)
     assert np.array_equal(gv, want_v), f"session {si}: V not bit-exact"
     # rows whose delta is 0 (the prefix before the first insert) keep their bits
@@ -49,11 +50,11 @@ def test_splice_c3_transposed_v_all_layers():
     T = case.w.spliced_len(s)
     got_k, got_v = gather_rows(case.kp, case.vp, case.h_pt[1], T, True)
     ins = s.inserts[0]
-    want_v = torch.cat([case.live_v[0][:, :ins.depth], case.blk_v[0][0],
-                        case.live_v[0][:, ins.depth:]], dim=1)
+    live_k, live_v = case.live(0)
+    want_v = torch.cat([live_v[:, :ins.depth], case.blk_v[0][0], live_v[:, ins.depth:]], dim=1)
     assert torch.equal(got_v.view(torch.int16), want_v.view(torch.int16))
     assert torch.equal(got_k[:, :ins.depth].view(torch.int16),
-                       case.live_k[0][:, :ins.depth].view(torch.int16))
+                       live_k[:, :ins.depth].view(torch.int16))
     for layers in ([0], [23], [47]):
         _check_session(case, 0, layers)
 
@@ -67,6 +68,29 @@ def test_splice_c4_sessions_shuffled_pages():
         _check_session(case, si, [0, 1])
 
 
+def test_splice_c4_full_size_sampled():
+    """32 sessions x 48 layers, four inserts each at random depths, shuffled pool
+    pages, one launch; V of every layer of the sampled sessions bit-exact, K of
+    sampled layers against the oracle."""
+    w = workload("c4")
+    case = SplicedCase(w, DEV, keep_live=False)
+    case.splice()
+    assert nexus.device_status() == nexus.OK
+    for si in (0, 13, 31):
+        s = w.sessions[si]
+        T = w.spliced_len(s)
+        _, got_v = gather_rows(case.kp, case.vp, case.h_pt[2 * si + 1], T, False)
+        _, live_v = case.live(si)
+        parts, cur = [], 0
+        for j, ins in enumerate(s.inserts):
+            parts += [live_v[:, cur:ins.depth], case.blk_v[si][j]]
+            cur = ins.depth
+        parts.append(live_v[:, cur:])
+        assert torch.equal(got_v.view(torch.int16), torch.cat(parts, dim=1).view(torch.int16))
+        del got_v, live_v, parts
+        _check_session(case, si, [0, 47])
+
+
 def test_splice_c5_full_size_sampled_layers():
     case = SplicedCase(workload("c5"), DEV)
     case.splice()
@@ -75,10 +99,10 @@ def test_splice_c5_full_size_sampled_layers():
     T = case.w.spliced_len(s)
     ins = s.inserts[0]
     got_k, got_v = gather_rows(case.kp, case.vp, case.h_pt[1], T, False)
-    want_v = torch.cat([case.live_v[0][:, :ins.depth], case.blk_v[0][0],
-                        case.live_v[0][:, ins.depth:]], dim=1)
+    _, live_v = case.live(0)
+    want_v = torch.cat([live_v[:, :ins.depth], case.blk_v[0][0], live_v[:, ins.depth:]], dim=1)
     assert torch.equal(got_v.view(torch.int16), want_v.view(torch.int16))
-    del got_k, got_v, want_v
+    del got_k, got_v, want_v, live_v
     for layers in ([0], [31]):
         _check_session(case, 0, layers)
 
