@@ -20,6 +20,7 @@ Retrieval-Decoupled Tool Routing for Agentic LLMs on Unified Memory"):
 * redecoded suffix length ceil(S * R / 100) ......................... Sec. V-A
 * scaled dot-product attention softmax(QK^T / sqrt(d)) V ............ Sec. III-A
 * R = 100 % is numerically a full prefill ........................... Sec. III-C
+* attention-logit soft-capping (models with token-innermost V) ....... Sec. V-B
 
 Readings taken where the paper is silent (each is listed in the design
 notes): NeoX half-split pairs (i, i + d/2) by default with GPT-J interleaved
@@ -206,12 +207,16 @@ def suffix_positions(T: int, R: int) -> np.ndarray:
     return np.arange(T - R, T, dtype=np.int64)
 
 
-def attention(q, k, v, q_pos, group: int):
+def attention(q, k, v, q_pos, group: int, softcap=None):
     """Causal GQA attention, the plain definition softmax(QK^T / sqrt(d)) V.
 
     q [R][Hq][d]; k, v [T][Hkv][d]; query t sees keys j <= q_pos[t]; query head
     h reads KV head h // group. Returns (o [R][Hq][d], lse [R][Hq]) with
-    lse = log sum_j exp(q.k_j / sqrt(d)) over the visible keys.
+    lse = log sum_j exp(s_j) over the visible keys, s_j = q.k_j / sqrt(d).
+
+    ``softcap`` (attention-logit soft-capping of the models whose V cache is
+    token-innermost, Sec. V-B): the scaled score s is replaced by
+    softcap * tanh(s / softcap) before the softmax.
     """
     q = np.asarray(q, dtype=np.float64)
     k = np.asarray(k, dtype=np.float64)
@@ -225,6 +230,8 @@ def attention(q, k, v, q_pos, group: int):
     for h in range(Hq):
         kv = h // group
         s = (q[:, h, :] @ k[:, kv, :].T) / math.sqrt(d)       # [R][T]
+        if softcap is not None:
+            s = softcap * np.tanh(s / softcap)
         s = np.where(visible, s, -np.inf)
         m = s.max(axis=1, keepdims=True)
         e = np.exp(s - m)

@@ -345,3 +345,32 @@ def pin_attention_split(attention):
         oc, lc = attention(q, kk, vv, pos - a, 2)
         acc += np.exp(lc - lse)[..., None] * oc
     assert np.max(np.abs(acc - o)) < 1e-12
+
+
+def pin_attention_softcap(attention):
+    """Soft-capped scores (Sec. V-B): a very large cap is plain attention; a key
+    with an enormous score saturates at +cap, so its weight is the closed form
+    e^cap / (e^cap + n_other); caps apply to the 1/sqrt(d)-scaled score."""
+    r = _rs(21)
+    R, T, d = 5, 30, 64
+    q = r.standard_normal((R, 4, d))
+    k = r.standard_normal((T, 2, d))
+    v = r.standard_normal((T, 2, d))
+    pos = np.arange(T - R, T)
+    o1, l1 = attention(q, k, v, pos, 2)
+    o2, l2 = attention(q, k, v, pos, 2, softcap=1.0e7)
+    assert np.max(np.abs(o1 - o2)) < 1e-9 and np.max(np.abs(l1 - l2)) < 1e-9
+    # saturation: key 0 aligned with an enormous query, the others orthogonal (score 0)
+    cap = 3.0
+    qq = np.zeros((1, 1, d)); qq[0, 0, 0] = 1.0e6
+    kk = np.zeros((8, 1, d)); kk[0, 0, 0] = 1.0; kk[1:, 0, 1] = 1.0
+    vv = np.zeros((8, 1, d)); vv[0, 0, 0] = 1.0
+    o, lse = attention(qq, kk, vv, [7], 1, softcap=cap)
+    w0 = math.exp(cap) / (math.exp(cap) + 7.0)
+    assert abs(o[0, 0, 0] - w0) < 1e-12
+    assert abs(lse[0, 0] - math.log(math.exp(cap) + 7.0)) < 1e-12
+    # the cap sees the scaled score: s = 2 / sqrt(d) gives cap * tanh(s / cap)
+    qq = np.zeros((1, 1, d)); qq[0, 0, 0] = 2.0
+    o, lse = attention(qq, kk, vv, [7], 1, softcap=cap)
+    s0 = cap * math.tanh((2.0 / math.sqrt(d)) / cap)
+    assert abs(lse[0, 0] - math.log(math.exp(s0) + 7.0)) < 1e-12

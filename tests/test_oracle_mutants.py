@@ -174,3 +174,26 @@ ATTN_MUTANTS = {
 def test_attention_mutants_caught(name):
     m = ATTN_MUTANTS[name]
     assert (_fails(P.pin_attention_library, m) or _fails(P.pin_attention_special, m))
+
+
+def test_softcap_mutants_caught():
+    def cap_before_scale(q, k, v, q_pos, group, softcap=None):
+        q = np.asarray(q, float); k = np.asarray(k, float); v = np.asarray(v, float)
+        R, Hq, d = q.shape
+        T = k.shape[0]
+        vis = np.arange(T)[None, :] <= np.asarray(q_pos)[:, None]
+        o = np.zeros((R, Hq, d)); lse = np.zeros((R, Hq))
+        for h in range(Hq):
+            s = q[:, h] @ k[:, h // group].T
+            if softcap is not None:
+                s = softcap * np.tanh(s / softcap)
+            s = np.where(vis, s / math.sqrt(d), -np.inf)
+            m = s.max(1, keepdims=True); e = np.exp(s - m); z = e.sum(1, keepdims=True)
+            o[:, h] = (e / z) @ v[:, h // group]; lse[:, h] = m[:, 0] + np.log(z[:, 0])
+        return o, lse
+
+    def cap_ignored(q, k, v, q_pos, group, softcap=None):
+        return oracle.attention(q, k, v, q_pos, group)
+
+    assert _fails(P.pin_attention_softcap, cap_before_scale)
+    assert _fails(P.pin_attention_softcap, cap_ignored)

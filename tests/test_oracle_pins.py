@@ -71,3 +71,7 @@ def test_bf16_widening():
     got = oracle.bf16_bits_to_f64(bits)
     assert np.array_equal(got, x.to(torch.float64).numpy())
     assert np.signbit(got[1])
+
+
+def test_attention_softcap():
+    P.pin_attention_softcap(oracle.attention)
