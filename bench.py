@@ -133,16 +133,17 @@ class ClockSampler:
 
 # --------------------------------------------------------------- workload
 class C5:
-    """Device-resident c5 workload and the library calls of one step."""
+    """Device-resident c5 workload and the library calls of one step (also used
+    with the c3 workload, whose cache keeps V token-innermost, for captures)."""
 
-    def __init__(self, dev, n_layers=48):
+    def __init__(self, dev, n_layers=48, name="c5"):
         import torch
 
         from paper_2608_20397_gb300 import nexus
         from paper_2608_20397_gb300.workloads import page_order, randn_bf16, workload
 
         self.torch, self.nexus = torch, nexus
-        w = workload("c5", n_layers=n_layers)
+        w = workload(name, n_layers=n_layers)
         self.w = w
         s = w.sessions[0]
         ins = s.inserts[0]
@@ -154,8 +155,10 @@ class C5:
         self.max_pages = -(-self.T // PAGE) + 1
         n_pages = -(-self.n_past // PAGE) + self.max_pages + 16
         self.pool = nexus.PagePool(n_pages, page_order(n_pages, w.seed, w.shuffle_pages))
+        self.vt = w.v_transposed
         self.kp = torch.zeros((L, n_pages, HKV, PAGE, D), dtype=torch.bfloat16, device=dev)
-        self.vp = torch.zeros_like(self.kp)
+        vshape = (L, n_pages, HKV, D, PAGE) if self.vt else (L, n_pages, HKV, PAGE, D)
+        self.vp = torch.zeros(vshape, dtype=torch.bfloat16, device=dev)
         h_pt = np.full((2, self.max_pages), -1, np.int32)
         npg = -(-self.n_past // PAGE)
         h_pt[0, :npg] = self.pool.alloc(npg)
@@ -166,10 +169,13 @@ class C5:
             k = randn_bf16((1, self.n_past, HKV, D), 500 + l, dev)
             v = randn_bf16((1, self.n_past, HKV, D), 600 + l, dev)
             self.kp[l, pg, :, pos % PAGE] = k[0]
-            self.vp[l, pg, :, pos % PAGE] = v[0]
+            if self.vt:
+                self.vp[l, pg, :, :, pos % PAGE] = v[0]
+            else:
+                self.vp[l, pg, :, pos % PAGE] = v[0]
         self.bk = randn_bf16((L, self.Lb, HKV, D), 700, dev)
         self.bv = randn_bf16((L, self.Lb, HKV, D), 701, dev)
-        self.cache = nexus.kv_cache(self.kp, self.vp, n_pages, L, HKV)
+        self.cache = nexus.kv_cache(self.kp, self.vp, n_pages, L, HKV, self.vt)
         self.blocks = [nexus.block(self.bk, self.bv, self.Lb, ins.base_pos, L, HKV)]
         new_pt, self.segs, _ = nexus.plan_splice(self.pool, h_pt[0], self.n_past, self.max_pages,
                                                  self.blocks, [(self.depth, 0)], 0, 1)
@@ -293,8 +299,11 @@ def main():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--layers", type=int, default=48, help="layers of the workload (48 = c5)")
-    ap.add_argument("--profile", choices=["reprefill", "splice", "suffix"], default=None,
+    ap.add_argument("--profile", choices=["reprefill", "reprefill-softcap", "splice", "suffix"],
+                    default=None,
                     help="run only this kernel of the step (small case for ncu captures)")
+    ap.add_argument("--workload", choices=["c5", "c3"], default="c5",
+                    help="workload of --profile runs (c3: token-innermost V cache)")
     args = ap.parse_args()
 
     rank = int(os.environ.get("RANK", "0"))
@@ -315,7 +324,9 @@ def main():
 
     from paper_2608_20397_gb300 import nexus
     nexus.lib()
-    wl = C5(dev, args.layers)
+    if args.profile is None and args.workload != "c5":
+        raise SystemExit("the timed step is the c5 workload; --workload only applies to --profile")
+    wl = C5(dev, args.layers, args.workload)
     stream = torch.cuda.current_stream()
     peaks, peak_kind = measured_peaks()
 
@@ -425,6 +436,11 @@ def _profile_only(wl, args, stream):
             nexus.reprefill(wl.cache, wl.d_pt, 2, wl.max_pages, [wl.n_past], wl.q_pre[:1],
                             wl.o_pre[:1], wl.lse_pre[:1], HQ, 0, 1, rows=[0], split_kv=1,
                             stream=stream)
+        elif args.profile == "reprefill-softcap":
+            nexus.suffix_attention_softcap(wl.cache, wl.d_pt, 2, wl.max_pages, [wl.n_past],
+                                           [wl.n_past], wl.q_pre[:1], wl.o_pre[:1],
+                                           wl.lse_pre[:1], HQ, 0, 1, rows=[0], split_kv=1,
+                                           softcap=50.0, stream=stream)
         else:
             nexus.suffix_attention(wl.cache, wl.d_pt, 2, wl.max_pages, [wl.T], [wl.R_split],
                                    wl.q_suf[:1], wl.o_suf[:1], wl.lse_suf[:1], HQ, 0, 1, rows=[1],
@@ -442,8 +458,14 @@ def _profile_only(wl, args, stream):
     b.record(stream)
     torch.cuda.synchronize()
     st = nexus.device_status(stream)
-    print(json.dumps({"profile": args.profile, "layers": wl.L, "ms_per_launch":
-                      a.elapsed_time(b) / args.steps, "status": nexus.status_string(st)}), flush=True)
+    ms = a.elapsed_time(b) / args.steps
+    rate = {"splice": f"{wl.splice_bytes / (ms * 1e-3) / 1e9:.1f} GB/s",
+            "reprefill": f"{wl.flops_pre / wl.L / (ms * 1e-3) / 1e12:.1f} TFLOP/s",
+            "reprefill-softcap": f"{wl.flops_pre / wl.L / (ms * 1e-3) / 1e12:.1f} TFLOP/s",
+            "suffix": f"{wl.flops_suf / wl.L / (ms * 1e-3) / 1e12:.1f} TFLOP/s"}[args.profile]
+    print(json.dumps({"profile": args.profile, "workload": args.workload, "layers": wl.L,
+                      "ms_per_launch": ms, "rate": rate, "status": nexus.status_string(st)}),
+          flush=True)
     if st != nexus.OK:
         raise SystemExit(1)
 

@@ -291,6 +291,21 @@ nexus_status nexus_suffix_attention(const nexus_kv_cache* cache,
                                     void* workspace, size_t workspace_bytes,
                                     nexus_stream stream);
 
+/* nexus_suffix_attention with attention-logit soft-capping, the attention of the
+ * models whose V cache is token-innermost (Sec. V-B): each scaled score s is
+ * replaced by softcap * tanh(s / softcap) before the softmax (LSE is over the
+ * capped scores). softcap > 0 (e.g. 50); NEXUS_EINVAL otherwise. Both V
+ * layouts are accepted. */
+nexus_status nexus_suffix_attention_softcap(const nexus_kv_cache* cache,
+                                            const int32_t* d_page_tables, int32_t n_rows,
+                                            int32_t max_pages, int32_t n_seqs,
+                                            const int32_t* h_rows, const int32_t* h_kv_len,
+                                            const int32_t* h_q_len, const void* q, void* out,
+                                            float* lse, int32_t n_q_heads, int32_t layer_begin,
+                                            int32_t layer_end, int32_t split_kv, void* workspace,
+                                            size_t workspace_bytes, float softcap,
+                                            nexus_stream stream);
+
 /* Full causal re-prefill: nexus_suffix_attention with q_len = kv_len (the
  * R = 100 % end point of Eq. 2, Sec. III-C). */
 nexus_status nexus_reprefill(const nexus_kv_cache* cache, const int32_t* d_page_tables,

@@ -204,6 +204,19 @@ __device__ __forceinline__ void tmem_st8(uint32_t taddr, const uint32_t (&r)[8])
                : "memory");
 }
 
+// tanh(x) = 1 - 2 / (e^(2x) + 1), from the exponential and reciprocal units;
+// absolute error about 4e-7, so a soft-capped logit cap * tanh(s / cap) errs by
+// ~4e-7 * cap (saturates correctly to +-1 for large |x|). `x2` is 2 x log2(e).
+__device__ __forceinline__ float tanh_from_exp2(float x2) {
+  const float e = ex2_approx(x2);
+  float r;
+  asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(r) : "f"(e + 1.f));
+  return fmaf(-2.f, r, 1.f);
+}
+
+// kSoftcap: attention-logit soft-capping (Sec. V-B): the scaled score s becomes
+// cap * tanh(s / cap) before the softmax.
+template <bool kSoftcap>
 __global__ void __launch_bounds__(kThreads, 1)
 attention_kernel(const __grid_constant__ AttnLaunch p, const __grid_constant__ AttnMaps maps) {
   extern __shared__ uint8_t smem_raw[];
@@ -435,7 +448,8 @@ attention_kernel(const __grid_constant__ AttnLaunch p, const __grid_constant__ A
     const int tok0_x = x ? w.tok0[1] : w.tok0[0];
     const bool active = x < n_q && n_tiles > 0;
     const bool row_valid = x < n_q && (r < G * p.tile_tokens) && (tr < ntok_x);
-    const float sc = p.scale_log2;
+    // log2-domain multiplier of a score (or of its tanh when soft-capped)
+    const float sc = kSoftcap ? p.softcap_out : p.scale_log2;
     float m_run = -INFINITY;                   // running max, log2-scaled units
     float l_run = 0.f;
     bool ok = true;
@@ -454,6 +468,10 @@ attention_kernel(const __grid_constant__ AttnLaunch p, const __grid_constant__ A
         for (int q = 0; q < 4; ++q)
 #pragma unroll
           for (int e = 0; e < 32; ++e) s[q * 32 + e] = __uint_as_float(v[q][e]);
+      }
+      if constexpr (kSoftcap) {
+#pragma unroll
+        for (int c = 0; c < BN; ++c) s[c] = tanh_from_exp2(s[c] * p.softcap_in);
       }
       const int lim = pos_r - (w.kt_begin + j) * BN;   // keys c <= lim are visible
       if (lim < BN - 1) {
@@ -615,12 +633,13 @@ __global__ void __launch_bounds__(128) combine_kernel(const __grid_constant__ At
 cudaError_t launch_attention(const AttnLaunch& p, const AttnMaps& maps, cudaStream_t stream) {
   if (p.total_tiles <= 0 || p.n_layers_call <= 0) return cudaSuccess;
   static_assert(kSmemBytes <= 227 * 1024, "shared memory budget");
-  cudaError_t e = cudaFuncSetAttribute(attention_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+  auto kernel = p.softcap_out > 0.f ? attention_kernel<true> : attention_kernel<false>;
+  cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        (int)kSmemBytes);
   if (e != cudaSuccess) return e;
   const dim3 grid((unsigned)p.total_tiles, (unsigned)p.n_kv_heads,
                   (unsigned)(p.n_layers_call * p.splits));
-  attention_kernel<<<grid, kThreads, kSmemBytes, stream>>>(p, maps);
+  kernel<<<grid, kThreads, kSmemBytes, stream>>>(p, maps);
   return cudaGetLastError();
 }
 

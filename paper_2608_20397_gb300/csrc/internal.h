@@ -101,6 +101,8 @@ struct AttnLaunch {
   int32_t v_transposed;
   int32_t total_tiles;      // CTAs per (KV head, layer, split): pairs of 128-row query tiles
   float scale_log2;         // log2(e) / sqrt(head_dim)
+  float softcap_in;         // soft-capping: 2 log2(e) / (sqrt(head_dim) cap)
+  float softcap_out;        // soft-capping: cap log2(e); 0 = no soft-capping
   int32_t tile_prefix[kMaxSeqs + 1];   // first CTA (tile pair) of each sequence
   AttnSeq seq[kMaxSeqs];
 };

@@ -295,8 +295,10 @@ nexus_status attention_impl(const nexus_kv_cache* c, const int32_t* d_pt, int32_
                             int32_t max_pages, int32_t n_seqs, const int32_t* h_rows,
                             const int32_t* kv_len, const int32_t* q_len, const void* q, void* out,
                             float* lse, int32_t n_q_heads, int32_t lb, int32_t le,
-                            int32_t split_kv, void* ws, size_t ws_bytes, cudaStream_t stream) {
+                            int32_t split_kv, void* ws, size_t ws_bytes, cudaStream_t stream,
+                            float softcap = 0.f) {
   nexus_status st = check_cache(c);
+  if (!(softcap >= 0.f) || !std::isfinite(softcap)) return NEXUS_EINVAL;
   if (st != NEXUS_OK) return st;
   if ((st = check_layers(c, lb, le)) != NEXUS_OK) return st;
   if (!d_pt || n_rows < 1 || max_pages < 1 || !q || !out) return NEXUS_EINVAL;
@@ -336,6 +338,11 @@ nexus_status attention_impl(const nexus_kv_cache* c, const int32_t* d_pt, int32_
   p->v_transposed = c->v_transposed;
   p->total_tiles = pl.total_tiles;
   p->scale_log2 = static_cast<float>(1.4426950408889634 / std::sqrt(static_cast<double>(kHeadDim)));
+  if (softcap > 0.f) {
+    p->softcap_in = static_cast<float>(2.0 * 1.4426950408889634 /
+                                       (std::sqrt(static_cast<double>(kHeadDim)) * softcap));
+    p->softcap_out = static_cast<float>(1.4426950408889634 * softcap);
+  }
   if (pl.splits > 1) {
     const size_t rows = static_cast<size_t>(pl.n_tok) * n_q_heads * (le - lb);
     p->part_o = static_cast<float*>(ws);
@@ -499,6 +506,18 @@ nexus_status nexus_suffix_attention(const nexus_kv_cache* cache, const int32_t* 
   return attention_impl(cache, d_page_tables, n_rows, max_pages, n_seqs, h_rows, h_kv_len, h_q_len,
                         q, out, lse, n_q_heads, layer_begin, layer_end, split_kv, workspace,
                         workspace_bytes, static_cast<cudaStream_t>(stream));
+}
+
+nexus_status nexus_suffix_attention_softcap(
+    const nexus_kv_cache* cache, const int32_t* d_page_tables, int32_t n_rows, int32_t max_pages,
+    int32_t n_seqs, const int32_t* h_rows, const int32_t* h_kv_len, const int32_t* h_q_len,
+    const void* q, void* out, float* lse, int32_t n_q_heads, int32_t layer_begin,
+    int32_t layer_end, int32_t split_kv, void* workspace, size_t workspace_bytes, float softcap,
+    nexus_stream stream) {
+  if (!(softcap > 0.f)) return NEXUS_EINVAL;
+  return attention_impl(cache, d_page_tables, n_rows, max_pages, n_seqs, h_rows, h_kv_len, h_q_len,
+                        q, out, lse, n_q_heads, layer_begin, layer_end, split_kv, workspace,
+                        workspace_bytes, static_cast<cudaStream_t>(stream), softcap);
 }
 
 nexus_status nexus_reprefill(const nexus_kv_cache* cache, const int32_t* d_page_tables,

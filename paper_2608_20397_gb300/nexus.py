@@ -101,6 +101,11 @@ _SIGS = {
                                          _i32p, _i32p, _i32p, c_void_p, c_void_p, c_void_p,
                                          c_int32, c_int32, c_int32, c_int32, c_void_p, c_size_t,
                                          c_void_p]),
+    "nexus_suffix_attention_softcap": (c_int32, [POINTER(KvCache), c_void_p, c_int32, c_int32,
+                                                 c_int32, _i32p, _i32p, _i32p, c_void_p,
+                                                 c_void_p, c_void_p, c_int32, c_int32, c_int32,
+                                                 c_int32, c_void_p, c_size_t, ctypes.c_float,
+                                                 c_void_p]),
     "nexus_reprefill": (c_int32, [POINTER(KvCache), c_void_p, c_int32, c_int32, c_int32, _i32p,
                                   _i32p, c_void_p, c_void_p, c_void_p, c_int32, c_int32, c_int32,
                                   c_int32, c_void_p, c_size_t, c_void_p]),
@@ -348,6 +353,20 @@ def suffix_attention(cache: KvCache, d_page_tables, n_rows: int, max_pages: int,
         rw[0] if rw else None, kv[0], ql[0], _ptr(q), _ptr(out), _ptr(lse), int(n_q_heads),
         int(layer_begin), int(layer_end), int(split_kv), _ptr(workspace), int(workspace_bytes),
         _stream(stream)))
+
+
+def suffix_attention_softcap(cache: KvCache, d_page_tables, n_rows: int, max_pages: int, kv_len,
+                             q_len, q, out, lse=None, n_q_heads: int = 40, layer_begin: int = 0,
+                             layer_end: int = 1, rows=None, split_kv: int = 0, workspace=None,
+                             workspace_bytes: int = 0, softcap: float = 50.0, stream=None):
+    kv = _i32(kv_len)
+    ql = _i32(q_len)
+    rw = _i32(rows)
+    _check("nexus_suffix_attention_softcap", lib().nexus_suffix_attention_softcap(
+        ctypes.byref(cache), _ptr(d_page_tables), int(n_rows), int(max_pages), len(kv[1]),
+        rw[0] if rw else None, kv[0], ql[0], _ptr(q), _ptr(out), _ptr(lse), int(n_q_heads),
+        int(layer_begin), int(layer_end), int(split_kv), _ptr(workspace), int(workspace_bytes),
+        float(softcap), _stream(stream)))
 
 
 def reprefill(cache: KvCache, d_page_tables, n_rows: int, max_pages: int, kv_len, q, out,

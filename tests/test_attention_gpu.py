@@ -50,13 +50,14 @@ def _run(cache, d_pt, max_pages, kv_lens, q_lens, q, Hq, L, split_kv=1, rows=Non
     return o, lse
 
 
-def _check(ks, vs, q, o, lse, kv_lens, q_lens, group, layer=0, what=""):
+def _check(ks, vs, q, o, lse, kv_lens, q_lens, group, layer=0, what="", softcap=None):
     off = 0
     for i, (T, R) in enumerate(zip(kv_lens, q_lens)):
         if R == 0:
             continue
         want_o, want_l = oracle.attention(f64(q[layer, off:off + R]), f64(ks[i][layer]),
-                                          f64(vs[i][layer]), oracle.suffix_positions(T, R), group)
+                                          f64(vs[i][layer]), oracle.suffix_positions(T, R), group,
+                                          softcap=softcap)
         assert_attn_close(f64(o[layer, off:off + R]), want_o, f64(lse[layer, off:off + R]), want_l,
                           f"{what} seq {i} T={T} R={R}")
         off += R
@@ -243,3 +244,49 @@ def test_end_to_end_c4_varlen_full_size():
                                               want_v[0, :kmax], pos, 5)
             assert_attn_close(f64(o[0, offs[si] + sel]), want_o, f64(lse[0, offs[si] + sel]),
                               want_l, f"c4 session {si} layer {layer}")
+
+
+# ------------------------------------------------ soft-capped attention (Sec. V-B)
+@pytest.mark.parametrize("cap,vt,split,qscale", [(50.0, True, 1, 1.0), (50.0, False, 1, 1.0),
+                                                 (5.0, True, 1, 8.0), (1.5, False, 1, 20.0),
+                                                 (30.0, True, 7, 1.0)])
+def test_softcap_attention(cap, vt, split, qscale):
+    kv, ql = [1500, 333], [300, 17]
+    cache, d_pt, mp, ks, vs, q = _direct_case(kv, ql, vt=vt, seed=int(cap) + split)
+    q = (q.float() * qscale).to(torch.bfloat16)       # larger scores: more of them saturate
+    o = torch.full_like(q, float("nan"))
+    lse = torch.full(q.shape[:3], float("nan"), dtype=torch.float32, device=DEV)
+    nbytes, _ = nexus.attention_workspace_size(kv, ql, 40, 8, 1, split)
+    ws = torch.empty(max(nbytes, 16), dtype=torch.uint8, device=DEV)
+    nexus.suffix_attention_softcap(cache, d_pt, 2, mp, kv, ql, q, o, lse, 40, 0, 1,
+                                   split_kv=split, workspace=ws, workspace_bytes=nbytes,
+                                   softcap=cap)
+    assert nexus.device_status() == nexus.OK
+    _check(ks, vs, q, o, lse, kv, ql, 5, what=f"softcap {cap}", softcap=cap)
+
+
+def test_end_to_end_c3_softcap():
+    """c3 (token-innermost V, 48 layers) with a Gemma-2-style cap of 50 over the
+    whole 2192-row suffix, sampled rows of two layers."""
+    w = workload("c3")
+    case = SplicedCase(w, DEV)
+    case.splice()
+    s0 = w.sessions[0]
+    T, R = w.spliced_len(s0), 2192
+    q = randn_bf16((1, R, 40, 128), 3300, DEV)
+    rows = np.sort(np.random.default_rng(33).choice(R, size=64, replace=False))
+    for layer in (0, 47):
+        o = torch.empty_like(q)
+        lse = torch.empty(q.shape[:3], dtype=torch.float32, device=DEV)
+        nexus.suffix_attention_softcap(case.cache, case.d_pt, case.n_rows, case.max_pages, [T],
+                                       [R], q, o, lse, 40, layer, layer + 1, rows=[1],
+                                       split_kv=1, softcap=50.0)
+        assert nexus.device_status() == nexus.OK
+        live_k, live_v = case.live(0)
+        want_k, want_v = oracle.splice_sequence(f64(live_k[[layer]]), f64(live_v[[layer]]),
+                                                case.inserts_f64(0, [layer]), w.rope_theta)
+        pos = oracle.suffix_positions(T, R)[rows]
+        want_o, want_l = oracle.attention(f64(q[0, rows]), want_k[0], want_v[0], pos, 5,
+                                          softcap=50.0)
+        assert_attn_close(f64(o[0, rows]), want_o, f64(lse[0, rows]), want_l,
+                          f"c3 softcap layer {layer}")

@@ -307,3 +307,11 @@ def test_workspace_size_and_split_choice():
     assert s == 1 and n == 0
     n, s = nexus.attention_workspace_size([34816], [64], 40, 8, 1, 7)
     assert s == 7 and n == 7 * 64 * 40 * 516
+
+
+def test_softcap_must_be_positive():
+    for cap in (0.0, -1.0, float("nan"), float("inf")):
+        with pytest.raises(nexus.NexusError) as e:
+            nexus.suffix_attention_softcap(_cache(), FAKE, 1, 8, [10], [5], FAKE, FAKE,
+                                           softcap=cap, stream=0)
+        assert e.value.code == nexus.EINVAL
