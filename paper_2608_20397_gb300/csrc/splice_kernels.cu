@@ -144,6 +144,10 @@ __global__ void __launch_bounds__(kThreads) splice_kernel(const __grid_constant_
   const bool do_v = (sg.flags & NEXUS_SEG_K_ONLY) == 0 && p.out_mode == kOutPool;
   const int64_t page_elems = (int64_t)H * kPageSize * kHeadDim;
   const int items = ns * H * 8;
+  // Block rows headed for a token-innermost V cache are loaded with K and staged
+  // in shared memory from registers, so their loads overlap K's.
+  const bool stage_from_regs = do_v && p.v_transposed && from_block &&
+                               items <= kItemsPerThread * kThreads;
 
   // ---- K (always row-major), and row-major V, through registers
   uint4 klo[kItemsPerThread], khi[kItemsPerThread], vlo[kItemsPerThread], vhi[kItemsPerThread];
@@ -176,7 +180,7 @@ __global__ void __launch_bounds__(kThreads) splice_kernel(const __grid_constant_
     src_pos_of[u] = sg.src_start + r;
     klo[u] = *reinterpret_cast<const uint4*>(sk + c * 8);
     khi[u] = *reinterpret_cast<const uint4*>(sk + 64 + c * 8);
-    if (do_v && !p.v_transposed) {
+    if ((do_v && !p.v_transposed) || stage_from_regs) {
       vlo[u] = *reinterpret_cast<const uint4*>(sv + c * 8);
       vhi[u] = *reinterpret_cast<const uint4*>(sv + 64 + c * 8);
     }
@@ -214,6 +218,12 @@ __global__ void __launch_bounds__(kThreads) splice_kernel(const __grid_constant_
       uint16_t* dv = p.v_pool + dst_off[u];
       *reinterpret_cast<uint4*>(dv) = vlo[u];
       *reinterpret_cast<uint4*>(dv + 64) = vhi[u];
+    } else if (stage_from_regs) {
+      const int h = (it >> 3) % H;
+      const int rl = it / (8 * H);
+      uint16_t* st = s_vstage + (slot0 + rl) * H * kHeadDim + h * kHeadDim + c * 8;
+      *reinterpret_cast<uint4*>(st) = vlo[u];
+      *reinterpret_cast<uint4*>(st + 64) = vhi[u];
     }
   }
   // Items past kItemsPerThread * kThreads (more than 8 KV heads) take a plain loop.
@@ -269,7 +279,34 @@ __global__ void __launch_bounds__(kThreads) splice_kernel(const __grid_constant_
   // ---- token-innermost V: stage [slot][head][d] in shared memory, then write
   // each (head, d) row of 16 slots as 32 contiguous bytes (Sec. V-B).
   const int hd_rows = H * kHeadDim;
-  if (from_block) {
+  if (!from_block && (sg.src_start + r0) % kPageSize == slot0) {
+    // Source and destination slots coincide (the rows moved by a multiple of
+    // 16): the piece is one page-to-page copy of token-innermost rows.
+    const int32_t spage =
+        p.page_tables[(int64_t)sg.src_row * p.max_pages + (sg.src_start + r0) / kPageSize];
+    const uint16_t* src = p.v_pool + ((int64_t)layer * p.n_pages + spage) * page_elems;
+    uint16_t* dst = p.v_pool + ((int64_t)layer * p.n_pages + dpage) * page_elems;
+    if (ns == kPageSize) {
+      const int vecs = (int)(page_elems / 8);
+      uint4 buf[4];
+      for (int i0 = threadIdx.x; i0 < vecs; i0 += 4 * kThreads) {
+#pragma unroll
+        for (int u = 0; u < 4; ++u)
+          if (i0 + u * kThreads < vecs) buf[u] = reinterpret_cast<const uint4*>(src)[i0 + u * kThreads];
+#pragma unroll
+        for (int u = 0; u < 4; ++u)
+          if (i0 + u * kThreads < vecs) reinterpret_cast<uint4*>(dst)[i0 + u * kThreads] = buf[u];
+      }
+    } else {
+      for (int hd = threadIdx.x; hd < hd_rows; hd += kThreads)
+        for (int s2 = slot0; s2 < slot0 + ns; ++s2)
+          dst[(int64_t)hd * kPageSize + s2] = src[(int64_t)hd * kPageSize + s2];
+    }
+    return;
+  }
+  if (stage_from_regs) {
+    // already staged by the register loop
+  } else if (from_block) {
     const int chunks = ns * H * 16;   // 16-byte chunks of the source rows
     for (int it = threadIdx.x; it < chunks; it += kThreads) {
       const int cc = it % (H * 16);
