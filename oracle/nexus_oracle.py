@@ -21,6 +21,7 @@ Retrieval-Decoupled Tool Routing for Agentic LLMs on Unified Memory"):
 * scaled dot-product attention softmax(QK^T / sqrt(d)) V ............ Sec. III-A
 * R = 100 % is numerically a full prefill ........................... Sec. III-C
 * attention-logit soft-capping (models with token-innermost V) ....... Sec. V-B
+* the re-decoded suffix tokens' fresh Q, K, V (projection, RoPE) ..... Sec. V-A, Sec. III-B
 
 Readings taken where the paper is silent (each is listed in the design
 notes): NeoX half-split pairs (i, i + d/2) by default with GPT-J interleaved
@@ -47,6 +48,7 @@ __all__ = [
     "paged_gather",
     "attention",
     "suffix_positions",
+    "qkv_recompute",
 ]
 
 
@@ -239,3 +241,32 @@ def attention(q, k, v, q_pos, group: int, softcap=None):
         o[:, h, :] = (e / z) @ v[:, kv, :]
         lse[:, h] = m[:, 0] + np.log(z[:, 0])
     return o, lse
+
+
+# --------------------------------------------------------------------------
+# Re-decoding the suffix: fresh Q, K, V of the invalidated tokens (Sec. V-A)
+# --------------------------------------------------------------------------
+def qkv_recompute(x, w_qkv, b_qkv, positions, n_q_heads: int, n_kv_heads: int,
+                  theta_base: float = 1.0e6, freq_scale: float = 1.0, rope_type: str = "neox"):
+    """Q, K, V of re-decoded tokens at the given positions (Sec. V-A, Sec. III-B).
+
+    x [R][hidden]; w_qkv [(Hq + 2 Hkv) d][hidden] (output features, input
+    features); b_qkv [(Hq + 2 Hkv) d] or None. y = x w_qkv^T + b is split, in
+    this order, into Q (Hq heads), K (Hkv heads) and V (Hkv heads) of d = 128
+    features; Q and K are rotated at each token's position, V is not.
+    Returns q [R][Hq][d], k [R][Hkv][d], v [R][Hkv][d].
+    """
+    x = np.asarray(x, dtype=np.float64)
+    w = np.asarray(w_qkv, dtype=np.float64)
+    y = x @ w.T
+    if b_qkv is not None:
+        y = y + np.asarray(b_qkv, dtype=np.float64)[None, :]
+    R = x.shape[0]
+    d = w.shape[0] // (n_q_heads + 2 * n_kv_heads)
+    q = y[:, : n_q_heads * d].reshape(R, n_q_heads, d)
+    k = y[:, n_q_heads * d: (n_q_heads + n_kv_heads) * d].reshape(R, n_kv_heads, d)
+    v = y[:, (n_q_heads + n_kv_heads) * d:].reshape(R, n_kv_heads, d)
+    pos = np.asarray(positions, dtype=np.float64)[:, None]
+    q = rope_rotate(q, pos, theta_base, freq_scale, rope_type)
+    k = rope_rotate(k, pos, theta_base, freq_scale, rope_type)
+    return q, k, v

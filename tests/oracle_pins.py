@@ -374,3 +374,32 @@ def pin_attention_softcap(attention):
     o, lse = attention(qq, kk, vv, [7], 1, softcap=cap)
     s0 = cap * math.tanh((2.0 / math.sqrt(d)) / cap)
     assert abs(lse[0, 0] - math.log(math.exp(s0) + 7.0)) < 1e-12
+
+
+def pin_qkv_recompute(qkv_recompute, rope_rotate):
+    """The re-decoded tokens' projection (Sec. V-A): a one-hot input row picks
+    column j of the weight plus the bias (at position 0, where RoPE is the
+    identity); Q heads come first, then K, then V; the map is affine in x; Q and
+    K at position p are the position-0 vectors rotated by p; V ignores position."""
+    r = _rs(22)
+    Hq, Hkv, d, hidden = 4, 2, 8, 6
+    out = (Hq + 2 * Hkv) * d
+    w = r.standard_normal((out, hidden))
+    b = r.standard_normal(out)
+    for j in range(hidden):
+        x = np.zeros((1, hidden)); x[0, j] = 1.0
+        q, k, v = qkv_recompute(x, w, b, [0], Hq, Hkv)
+        col = w[:, j] + b
+        assert np.allclose(q.reshape(-1), col[: Hq * d], atol=1e-14, rtol=0)
+        assert np.allclose(k.reshape(-1), col[Hq * d: (Hq + Hkv) * d], atol=1e-14, rtol=0)
+        assert np.allclose(v.reshape(-1), col[(Hq + Hkv) * d:], atol=1e-14, rtol=0)
+    x1, x2 = r.standard_normal((2, 3, hidden))
+    pos = np.array([5, 70, 3000])
+    f = lambda x: qkv_recompute(x, w, None, pos, Hq, Hkv)
+    for a, b2, c in zip(f(x1 + x2), f(x1), f(x2)):
+        assert np.max(np.abs(a - b2 - c)) < 1e-11
+    q0, k0, v0 = qkv_recompute(x1, w, b, [0, 0, 0], Hq, Hkv)
+    qp, kp, vp = qkv_recompute(x1, w, b, pos, Hq, Hkv)
+    assert np.max(np.abs(qp - rope_rotate(q0, pos[:, None]))) < 1e-11
+    assert np.max(np.abs(kp - rope_rotate(k0, pos[:, None]))) < 1e-11
+    assert np.array_equal(vp, v0)

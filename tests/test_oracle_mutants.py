@@ -197,3 +197,24 @@ def test_softcap_mutants_caught():
 
     assert _fails(P.pin_attention_softcap, cap_before_scale)
     assert _fails(P.pin_attention_softcap, cap_ignored)
+
+
+def test_qkv_mutants_caught():
+    def transposed_weight(x, w, b, positions, Hq, Hkv, *a, **kw):
+        w = np.asarray(w)
+        wt = w.reshape(-1)[: w.size].reshape(w.shape[1], w.shape[0]).T   # a mis-strided read
+        return oracle.qkv_recompute(x, wt, b, positions, Hq, Hkv)
+
+    def kv_swapped(x, w, b, positions, Hq, Hkv, *a, **kw):
+        q, k, v = oracle.qkv_recompute(x, w, b, positions, Hq, Hkv)
+        return q, v, k
+
+    def no_bias(x, w, b, positions, Hq, Hkv, *a, **kw):
+        return oracle.qkv_recompute(x, w, None, positions, Hq, Hkv)
+
+    def v_rotated(x, w, b, positions, Hq, Hkv, *a, **kw):
+        q, k, v = oracle.qkv_recompute(x, w, b, positions, Hq, Hkv)
+        return q, k, oracle.rope_rotate(v, np.asarray(positions)[:, None])
+
+    for mut in (transposed_weight, kv_swapped, no_bias, v_rotated):
+        assert _fails(P.pin_qkv_recompute, mut, oracle.rope_rotate), mut.__name__

@@ -75,3 +75,7 @@ def test_bf16_widening():
 
 def test_attention_softcap():
     P.pin_attention_softcap(oracle.attention)
+
+
+def test_qkv_recompute():
+    P.pin_qkv_recompute(oracle.qkv_recompute, oracle.rope_rotate)
