@@ -299,7 +299,8 @@ def main():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--layers", type=int, default=48, help="layers of the workload (48 = c5)")
-    ap.add_argument("--profile", choices=["reprefill", "reprefill-softcap", "splice", "suffix"],
+    ap.add_argument("--profile", choices=["reprefill", "reprefill-softcap", "splice", "suffix",
+                                          "qkv"],
                     default=None,
                     help="run only this kernel of the step (small case for ncu captures)")
     ap.add_argument("--workload", choices=["c5", "c3"], default="c5",
@@ -427,9 +428,26 @@ def _profile_only(wl, args, stream):
     for ncu captures; prints the mean CUDA-event time per launch."""
     import torch
     nexus = wl.nexus
+    if args.profile == "qkv":
+        # Fresh Q, K, V of the re-decoded tokens of one layer: the 100 % suffix
+        # of the spliced span (c3: 2192 tokens) or the whole context of the
+        # re-prefill (c5: 32768 tokens).
+        from paper_2608_20397_gb300.workloads import HIDDEN, qkv_weights, randn_bf16
+        if args.workload == "c3":
+            qkv_kv, qkv_n, qkv_row = wl.T, wl.w.sessions[0].suffix_span, 1
+        else:
+            qkv_kv, qkv_n, qkv_row = wl.n_past, wl.n_past, 0
+        dev = wl.kp.device
+        qkv_x = randn_bf16((qkv_n, HIDDEN), 1000, dev)
+        qkv_w, qkv_b = qkv_weights(HQ + 2 * HKV, HIDDEN, 1001, dev)
+        qkv_q = torch.empty((qkv_n, HQ, D), dtype=torch.bfloat16, device=dev)
+        qkv_flops = 2.0 * qkv_n * HIDDEN * (HQ + 2 * HKV) * D
 
     def one():
-        if args.profile == "splice":
+        if args.profile == "qkv":
+            nexus.suffix_qkv(wl.cache, wl.d_pt, 2, wl.max_pages, [qkv_kv], [qkv_n], qkv_x, qkv_w,
+                             qkv_b, qkv_q, layer=0, n_q_heads=HQ, rows=[qkv_row], stream=stream)
+        elif args.profile == "splice":
             nexus.splice_kv(wl.cache, wl.d_pt, None, 2, wl.max_pages, wl.blocks, wl.segs, 0, wl.L,
                             stream)
         elif args.profile == "reprefill":
@@ -459,6 +477,14 @@ def _profile_only(wl, args, stream):
     torch.cuda.synchronize()
     st = nexus.device_status(stream)
     ms = a.elapsed_time(b) / args.steps
+    if args.profile == "qkv":
+        print(json.dumps({"profile": "qkv", "workload": args.workload, "tokens": qkv_n,
+                          "ms_per_launch": ms,
+                          "rate": f"{qkv_flops / (ms * 1e-3) / 1e12:.1f} TFLOP/s",
+                          "status": nexus.status_string(st)}), flush=True)
+        if st != nexus.OK:
+            raise SystemExit(1)
+        return
     rate = {"splice": f"{wl.splice_bytes / (ms * 1e-3) / 1e9:.1f} GB/s",
             "reprefill": f"{wl.flops_pre / wl.L / (ms * 1e-3) / 1e12:.1f} TFLOP/s",
             "reprefill-softcap": f"{wl.flops_pre / wl.L / (ms * 1e-3) / 1e12:.1f} TFLOP/s",

@@ -18,6 +18,9 @@
  *                            Sec. III-A
  *   nexus_reprefill          the same with R = T: the full re-prefill that
  *                            R(n_past) = 100 % amounts to (Sec. III-C)
+ *   nexus_suffix_qkv         fresh Q, K, V of the re-decoded suffix tokens:
+ *                            QKV projection, RoPE at the new positions, K/V
+ *                            written into the paged cache (Sec. V-A, Sec. III-B)
  *   nexus_recompute_pct, nexus_redecode_len, nexus_check_splice
  *                            the depth-adaptive policy of Eq. 2 and the
  *                            splice threshold P (Sec. III-B, Sec. III-C)
@@ -144,8 +147,9 @@ int32_t nexus_version(void);
 
 /* Synchronises `stream`, then reports NEXUS_ETIMEOUT if any kernel of this
  * library on the current device gave up a bounded wait since the last call
- * (and clears that record), NEXUS_ECUDA if the stream reports an error,
- * else NEXUS_OK. */
+ * (and clears that record), NEXUS_ERANGE if nexus_suffix_qkv met a page id
+ * outside the pool (and skipped that token's cache write), NEXUS_ECUDA if the
+ * stream reports an error, else NEXUS_OK. */
 nexus_status nexus_device_status(nexus_stream stream);
 
 /* ---------------------------------------------------------------- policy */
@@ -314,6 +318,40 @@ nexus_status nexus_reprefill(const nexus_kv_cache* cache, const int32_t* d_page_
                              void* out, float* lse, int32_t n_q_heads, int32_t layer_begin,
                              int32_t layer_end, int32_t split_kv, void* workspace,
                              size_t workspace_bytes, nexus_stream stream);
+
+/* ------------------------------------------------- suffix Q/K/V recompute */
+/* The re-decode half of stitching the seam (Sec. V-A): after the splice, the
+ * last q_len[s] positions of each sequence are invalidated and re-decoded, which
+ * gives each of those tokens a fresh query, key and value. For one layer this
+ * computes, per token, y = x W^T + b, splits y into n_q_heads query heads, then
+ * n_kv_heads key heads, then n_kv_heads value heads (128 features each), rotates
+ * the query and key heads at the token's position (RoPE of Sec. III-B with the
+ * cache's parameters), writes the queries to q_out and the keys and values into
+ * the token's slot of the paged cache at `layer` (either V layout, Sec. V-B).
+ *   sequences   token t of sequence s (t < q_len[s]) sits at position
+ *               kv_len[s] - q_len[s] + t of page-table row h_rows[s] (h_rows
+ *               NULL: row s); its input is row q_off[s] + t of x, where
+ *               q_off[s] = sum of the earlier q_len
+ *   x           device bf16 [sum of q_len][hidden] (the layer's normalised
+ *               hidden states of the re-decoded tokens); hidden a multiple of 8
+ *   w_qkv       device bf16 [(n_q_heads + 2 n_kv_heads) * 128][hidden]
+ *   b_qkv       device float [(n_q_heads + 2 n_kv_heads) * 128], or NULL
+ *   q_out       device bf16 [sum of q_len][n_q_heads][128], the layout the
+ *               attention calls read their queries in
+ *   h_page_tables  host copy of the page tables (nullable): when given, every
+ *               written page is checked to lie in the pool (NEXUS_ERANGE) and
+ *               no two tokens may write one slot (NEXUS_EOVERLAP); without it
+ *               the kernel skips writes to a page id outside the pool and
+ *               nexus_device_status reports NEXUS_ERANGE
+ * Products accumulate in float32 on the tensor cores; the bias, the rotation
+ * (angles reduced to one float ulp) and the bf16 rounding of the stores follow.
+ * kv_len <= 2^24 (NEXUS_ERANGE). Writes nothing outside q_out and those slots. */
+nexus_status nexus_suffix_qkv(const nexus_kv_cache* cache, const int32_t* d_page_tables,
+                              const int32_t* h_page_tables, int32_t n_rows, int32_t max_pages,
+                              int32_t n_seqs, const int32_t* h_rows, const int32_t* h_kv_len,
+                              const int32_t* h_q_len, const void* x, int32_t hidden,
+                              const void* w_qkv, const float* b_qkv, int32_t n_q_heads,
+                              int32_t layer, void* q_out, nexus_stream stream);
 
 /* Bytes of workspace nexus_suffix_attention needs for these arguments
  * (0 when no split is used). *splits_out (nullable) receives the partition

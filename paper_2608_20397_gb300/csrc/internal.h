@@ -118,4 +118,39 @@ cudaError_t launch_attn_combine(const AttnLaunch& p, cudaStream_t stream);
 // Reads and clears the timeout record of the current device.
 cudaError_t attention_take_timeout(unsigned int* flag, cudaStream_t stream);
 
+// ------------------------------------------------- suffix Q/K/V recompute
+struct QkvLaunch {
+  const int32_t* page_tables;
+  const float* bias;        // nullable, [n_heads * 128]
+  uint16_t* q_out;          // [n_tok][n_q_heads][128]
+  uint16_t* k_pool;
+  uint16_t* v_pool;
+  int64_t n_pages;
+  int32_t max_pages;
+  int32_t n_q_heads;
+  int32_t n_kv_heads;
+  int32_t n_heads;          // n_q_heads + 2 n_kv_heads
+  int32_t layer;
+  int32_t v_transposed;
+  int32_t rope_gptj;
+  int32_t n_tok;            // packed tokens (sum of q_len)
+  int32_t k_blocks;         // ceil(hidden / 64)
+  int32_t n_tiles;          // 256-feature tiles: ceil(n_heads / 2)
+  int32_t total_tiles;      // ceil(n_tok / 128) * n_tiles
+  int32_t n_seqs;
+  float inv_freq_hi[kHeadDim / 2];   // theta_i / pi = hi + lo
+  float inv_freq_lo[kHeadDim / 2];
+  AttnSeq seq[kMaxSeqs];
+};
+
+struct QkvMaps {
+  CUtensorMap x;            // [n_tok][hidden], box 128 x 64
+  CUtensorMap w;            // [n_heads * 128][hidden], box 256 x 64
+};
+
+cudaError_t launch_qkv(const QkvLaunch& p, const QkvMaps& maps, int grid, cudaStream_t stream);
+// Reads and clears the device records of the Q/K/V kernel: a wait that gave up,
+// a page id outside the pool.
+cudaError_t qkv_take_status(unsigned int* timeout, unsigned int* bad_page, cudaStream_t stream);
+
 }  // namespace nexus

@@ -235,6 +235,21 @@ bool encode_4d(CUtensorMap* m, const void* base, const uint64_t dims[4], const u
   return r == CUDA_SUCCESS;
 }
 
+bool encode_2d_sw128(CUtensorMap* m, const void* base, uint64_t inner, uint64_t outer,
+                     uint32_t box_outer) {
+  auto enc = tensor_map_encoder();
+  if (!enc) return false;
+  const cuuint64_t dims[2] = {inner, outer};
+  const cuuint64_t strides[1] = {inner * 2};
+  const cuuint32_t box[2] = {64, box_outer};
+  const cuuint32_t elem[2] = {1, 1};
+  const CUresult r = enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims,
+                         strides, box, elem, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                         CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                         CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
 struct AttnPlan {
   int32_t total_tiles = 0;
   int32_t n_tok = 0;
@@ -399,12 +414,14 @@ nexus_status attention_impl(const nexus_kv_cache* c, const int32_t* d_pt, int32_
 extern "C" {
 
 nexus_status nexus_device_status(nexus_stream stream) {
-  unsigned int flag = 0;
-  if (attention_take_timeout(&flag, static_cast<cudaStream_t>(stream)) != cudaSuccess) {
+  unsigned int flag = 0, qkv_timeout = 0, bad_page = 0;
+  if (attention_take_timeout(&flag, static_cast<cudaStream_t>(stream)) != cudaSuccess ||
+      qkv_take_status(&qkv_timeout, &bad_page, static_cast<cudaStream_t>(stream)) != cudaSuccess) {
     cudaGetLastError();
     return NEXUS_ECUDA;
   }
-  return flag ? NEXUS_ETIMEOUT : NEXUS_OK;
+  if (flag || qkv_timeout) return NEXUS_ETIMEOUT;
+  return bad_page ? NEXUS_ERANGE : NEXUS_OK;
 }
 
 nexus_status nexus_splice_kv(const nexus_kv_cache* cache, const int32_t* d_page_tables,
@@ -529,6 +546,95 @@ nexus_status nexus_reprefill(const nexus_kv_cache* cache, const int32_t* d_page_
   return attention_impl(cache, d_page_tables, n_rows, max_pages, n_seqs, h_rows, h_kv_len, h_kv_len,
                         q, out, lse, n_q_heads, layer_begin, layer_end, split_kv, workspace,
                         workspace_bytes, static_cast<cudaStream_t>(stream));
+}
+
+nexus_status nexus_suffix_qkv(const nexus_kv_cache* cache, const int32_t* d_page_tables,
+                              const int32_t* h_page_tables, int32_t n_rows, int32_t max_pages,
+                              int32_t n_seqs, const int32_t* h_rows, const int32_t* h_kv_len,
+                              const int32_t* h_q_len, const void* x, int32_t hidden,
+                              const void* w_qkv, const float* b_qkv, int32_t n_q_heads,
+                              int32_t layer, void* q_out, nexus_stream stream) {
+  nexus_status st = check_cache(cache);
+  if (st != NEXUS_OK) return st;
+  if (layer < 0 || layer >= cache->n_layers) return NEXUS_ERANGE;
+  if (!d_page_tables || n_rows < 1 || max_pages < 1 || !x || !w_qkv || !q_out) return NEXUS_EINVAL;
+  if (n_seqs < 1 || n_seqs > kMaxSeqs || !h_kv_len || !h_q_len) return NEXUS_EINVAL;
+  if (n_q_heads < 1 || n_q_heads > 256 || hidden < 1) return NEXUS_EINVAL;
+  if (hidden % 8 != 0 || !aligned16(x) || !aligned16(w_qkv) || !aligned16(q_out) ||
+      (b_qkv && !aligned16(b_qkv)))
+    return NEXUS_ELAYOUT;
+  const int64_t cap = static_cast<int64_t>(max_pages) * kPageSize;
+  int64_t n_tok = 0;
+  for (int32_t s = 0; s < n_seqs; ++s) {
+    const int32_t row = h_rows ? h_rows[s] : s;
+    if (h_q_len[s] < 0 || h_kv_len[s] < h_q_len[s]) return NEXUS_EINVAL;
+    if (row < 0 || row >= n_rows || h_kv_len[s] > cap || h_kv_len[s] > (1 << 24))
+      return NEXUS_ERANGE;
+    n_tok += h_q_len[s];
+  }
+  const int32_t n_heads = n_q_heads + 2 * cache->n_kv_heads;
+  const int64_t n_tiles = (n_heads + 1) / 2;
+  const int64_t total = (n_tok + 127) / 128 * n_tiles;
+  if (n_tok > 0x7FFFFFFF || total > 0x7FFFFFFF) return NEXUS_ERANGE;
+  if (h_page_tables) {
+    // Every written slot lies in the pool and no two tokens share one.
+    std::vector<int64_t> slots;
+    slots.reserve(static_cast<size_t>(n_tok));
+    for (int32_t s = 0; s < n_seqs; ++s) {
+      const int32_t* pt = h_page_tables + static_cast<int64_t>(h_rows ? h_rows[s] : s) * max_pages;
+      for (int32_t pos = h_kv_len[s] - h_q_len[s]; pos < h_kv_len[s]; ++pos) {
+        const int32_t page = pt[pos / kPageSize];
+        if (page < 0 || page >= cache->n_pages) return NEXUS_ERANGE;
+        slots.push_back(static_cast<int64_t>(page) * kPageSize + pos % kPageSize);
+      }
+    }
+    std::sort(slots.begin(), slots.end());
+    if (std::adjacent_find(slots.begin(), slots.end()) != slots.end()) return NEXUS_EOVERLAP;
+  }
+  if (n_tok == 0) return NEXUS_OK;
+
+  std::unique_ptr<QkvLaunch> p(new QkvLaunch());
+  std::memset(p.get(), 0, sizeof(QkvLaunch));
+  p->page_tables = d_page_tables;
+  p->bias = b_qkv;
+  p->q_out = static_cast<uint16_t*>(q_out);
+  p->k_pool = static_cast<uint16_t*>(cache->k_pool);
+  p->v_pool = static_cast<uint16_t*>(cache->v_pool);
+  p->n_pages = cache->n_pages;
+  p->max_pages = max_pages;
+  p->n_q_heads = n_q_heads;
+  p->n_kv_heads = cache->n_kv_heads;
+  p->n_heads = n_heads;
+  p->layer = layer;
+  p->v_transposed = cache->v_transposed;
+  p->rope_gptj = cache->rope_type == NEXUS_ROPE_GPTJ;
+  p->n_tok = static_cast<int32_t>(n_tok);
+  p->k_blocks = (hidden + 63) / 64;
+  p->n_tiles = static_cast<int32_t>(n_tiles);
+  p->total_tiles = static_cast<int32_t>(total);
+  p->n_seqs = n_seqs;
+  double inv[kHeadDim / 2];
+  fill_inv_freq_over_pi(cache, inv);
+  for (int i = 0; i < kHeadDim / 2; ++i) {
+    p->inv_freq_hi[i] = static_cast<float>(inv[i]);
+    p->inv_freq_lo[i] = static_cast<float>(inv[i] - static_cast<double>(p->inv_freq_hi[i]));
+  }
+  int32_t off = 0;
+  for (int32_t s = 0; s < n_seqs; ++s) {
+    p->seq[s].kv_len = h_kv_len[s];
+    p->seq[s].q_len = h_q_len[s];
+    p->seq[s].q_off = off;
+    p->seq[s].pt_row = h_rows ? h_rows[s] : s;
+    off += h_q_len[s];
+  }
+  QkvMaps maps;
+  if (!encode_2d_sw128(&maps.x, x, static_cast<uint64_t>(hidden), static_cast<uint64_t>(n_tok), 128) ||
+      !encode_2d_sw128(&maps.w, w_qkv, static_cast<uint64_t>(hidden),
+                       static_cast<uint64_t>(n_heads) * kHeadDim, 256))
+    return NEXUS_ECUDA;
+  const int grid = static_cast<int>(std::min<int64_t>(total, num_sms()));
+  return launch_qkv(*p, maps, grid, static_cast<cudaStream_t>(stream)) == cudaSuccess ? NEXUS_OK
+                                                                                      : NEXUS_ECUDA;
 }
 
 size_t nexus_attention_workspace_size(int32_t n_seqs, const int32_t* h_kv_len,

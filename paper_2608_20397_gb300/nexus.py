@@ -115,6 +115,9 @@ _SIGS = {
                                                  c_int32, _i32p, _i32p, _i32p, c_void_p,
                                                  c_void_p, c_void_p, c_int32, c_int32, c_int32,
                                                  c_int32, c_void_p]),
+    "nexus_suffix_qkv": (c_int32, [POINTER(KvCache), c_void_p, _i32p, c_int32, c_int32, c_int32,
+                                   _i32p, _i32p, _i32p, c_void_p, c_int32, c_void_p, c_void_p,
+                                   c_int32, c_int32, c_void_p, c_void_p]),
 }
 EXPORTED = tuple(_SIGS)
 
@@ -398,3 +401,20 @@ def suffix_attention_noalloc(cache: KvCache, d_page_tables, n_rows: int, max_pag
         ctypes.byref(cache), _ptr(d_page_tables), int(n_rows), int(max_pages), len(kv[1]),
         rw[0] if rw else None, kv[0], ql[0], _ptr(q), _ptr(out), _ptr(lse), int(n_q_heads),
         int(layer_begin), int(layer_end), int(split_kv), _stream(stream)))
+
+
+def suffix_qkv(cache: KvCache, d_page_tables, n_rows: int, max_pages: int, kv_len, q_len, x,
+               w_qkv, b_qkv, q_out, layer: int = 0, n_q_heads: int = 40, rows=None,
+               h_page_tables=None, hidden: Optional[int] = None, stream=None):
+    """Fresh Q, K, V of the re-decoded suffix tokens of one layer (see nexus.h):
+    x [sum q_len][hidden] bf16, w_qkv [(Hq + 2 Hkv) 128][hidden] bf16, b_qkv float
+    or None; Q goes to q_out [sum q_len][Hq][128], K and V into the cache."""
+    kv = _i32(kv_len)
+    ql = _i32(q_len)
+    rw = _i32(rows)
+    hpt = _i32(h_page_tables)
+    _check("nexus_suffix_qkv", lib().nexus_suffix_qkv(
+        ctypes.byref(cache), _ptr(d_page_tables), hpt[0] if hpt else None, int(n_rows),
+        int(max_pages), len(kv[1]), rw[0] if rw else None, kv[0], ql[0], _ptr(x),
+        int(hidden if hidden is not None else x.shape[-1]), _ptr(w_qkv), _ptr(b_qkv), int(n_q_heads),
+        int(layer), _ptr(q_out), _stream(stream)))

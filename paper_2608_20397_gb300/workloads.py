@@ -27,6 +27,12 @@ Named workloads (Hq = 40, Hkv = 8, d = 128, 16-token pages):
 * ``c5``  48 layers, n_past 32768, one 2048-token block at depth 30000; a full
   causal re-prefill of the 32768-token context and a 64-query suffix over the
   34816-token spliced cache.
+
+Re-decoded suffix tokens (fresh Q, K, V): hidden states x ~ N(0, 1) bf16 of
+width 5120; the fused QKV weight [(40 + 2 * 8) * 128][5120] is N(0, 1) bf16
+scaled by 2^-6 (exact in bf16), so each projected feature has a standard
+deviation near 1.1, as in a trained layer after its input norm; the bias is
+float32 N(0, 1) / 2.
 """
 from __future__ import annotations
 
@@ -37,6 +43,7 @@ from typing import List, Optional
 import numpy as np
 import torch
 
+HIDDEN = 5120
 N_Q_HEADS = 40
 N_KV_HEADS = 8
 HEAD_DIM = 128
@@ -147,3 +154,14 @@ def randn_bf16(shape, seed: int, device="cpu") -> torch.Tensor:
         out[i0:i1] = torch.randn((i1 - i0,) + shape[1:], generator=g, device=device,
                                  dtype=torch.float32).to(torch.bfloat16)
     return out
+
+
+def qkv_weights(n_heads: int, hidden: int, seed: int, device="cpu", bias: bool = True):
+    """Fused QKV weight [n_heads * 128][hidden] (bf16) and bias (float32 or None)."""
+    w = randn_bf16((n_heads * HEAD_DIM, hidden), seed, device) * (2.0 ** -6)
+    b = None
+    if bias:
+        g = torch.Generator(device=device)
+        g.manual_seed(int(seed) * 1_000_003 + 7)
+        b = torch.randn((n_heads * HEAD_DIM,), generator=g, device=device, dtype=torch.float32) * 0.5
+    return w, b

@@ -315,3 +315,34 @@ def test_softcap_must_be_positive():
             nexus.suffix_attention_softcap(_cache(), FAKE, 1, 8, [10], [5], FAKE, FAKE,
                                            softcap=cap, stream=0)
         assert e.value.code == nexus.EINVAL
+
+
+def test_qkv_argument_checks():
+    c = _cache()
+    def call(kv=(40,), ql=(8,), hidden=64, x=FAKE, layer=0, hpt=None, rows=None, max_pages=8,
+             n_rows=1, bias=None):
+        nexus.suffix_qkv(c, FAKE, n_rows, max_pages, list(kv), list(ql), x, FAKE, bias, FAKE,
+                         layer=layer, rows=rows, h_page_tables=hpt, hidden=hidden, stream=0)
+
+    def code(**kw):
+        with pytest.raises(nexus.NexusError) as e:
+            call(**kw)
+        return e.value.code
+
+    assert code(ql=(41,)) == nexus.EINVAL                 # q_len > kv_len
+    assert code(kv=(200,)) == nexus.ERANGE                # beyond the page table
+    assert code(layer=2) == nexus.ERANGE                  # the cache has two layers
+    assert code(hidden=60) == nexus.ELAYOUT               # rows of x not 16-byte multiples
+    assert code(x=FAKE + 8) == nexus.ELAYOUT              # misaligned x
+    assert code(bias=FAKE + 4) == nexus.ELAYOUT           # misaligned bias
+    assert code(hidden=0) == nexus.EINVAL
+    assert code(rows=[1]) == nexus.ERANGE                 # page-table row outside the table
+    assert code(kv=((1 << 24) + 1,), max_pages=(1 << 20) + 1) == nexus.ERANGE   # float positions
+    pt = np.arange(16, dtype=np.int32).reshape(2, 8)
+    bad = pt.copy()
+    bad[0, 2] = 64                                        # pool has 64 pages
+    assert code(hpt=bad, n_rows=2) == nexus.ERANGE
+    shared = pt.copy()
+    shared[1, 2] = shared[0, 2]                           # both rows write page 2's slots
+    assert code(kv=(40, 40), ql=(8, 8), rows=[0, 1], hpt=shared, n_rows=2) == nexus.EOVERLAP
+    call(kv=(40, 40), ql=(0, 0), rows=[0, 1], hpt=pt, n_rows=2)   # nothing to do: no launch
