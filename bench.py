@@ -14,7 +14,9 @@ bf16, 16-token pages):
 
 The printed metric is attention TFLOP/s over the whole step (algorithmic,
 causal-visible flops 4 d Hq (R (T - R) + R (R + 1) / 2) per layer), with the
-splice GB/s (8192 algorithmic bytes per moved token-layer) beside it.
+splice GB/s (8192 algorithmic bytes per moved token-layer) beside it. The fresh
+Q/K/V of re-decoded tokens (projection + RoPE + cache write) is timed apart from
+the step under "qkv_recompute" (2 x 5120 x 7168 flops per token).
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
 
@@ -298,6 +300,8 @@ def main():
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-qkv", action="store_true",
+                    help="skip the separate timing of the suffix Q/K/V recompute")
     ap.add_argument("--layers", type=int, default=48, help="layers of the workload (48 = c5)")
     ap.add_argument("--profile", choices=["reprefill", "reprefill-softcap", "splice", "suffix",
                                           "qkv"],
@@ -391,6 +395,11 @@ def main():
     if not args.no_e2e:
         e2e = _e2e(wl, stream, args, barrier, world, dist, dev)
 
+    qkv = None
+    if not args.no_qkv:
+        qkv = _qkv_measure(wl, stream, peaks, peak_kind,
+                           with_oracle=rank == 0 and world == 1 and not args.no_cpu_baseline)
+
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         f64 = lambda t: t.float().cpu().double().numpy()
@@ -415,7 +424,7 @@ def main():
             "splice_gbs": splice_gbs, "splice_ms": splice_ms, "reprefill_ms": pre_ms,
             "suffix_ms": suf_ms, "suffix_tflops": suf_tflops,
             "roofline": roofline, "roofline_splice": roofline_splice,
-            "e2e": e2e, "cpu_baseline": cpu, "clocks": clocks,
+            "e2e": e2e, "cpu_baseline": cpu, "clocks": clocks, "qkv_recompute": qkv,
             "gpu_launches": wl.launches_per_step * args.steps,
         }
         print(json.dumps(line), flush=True)
@@ -494,6 +503,62 @@ def _profile_only(wl, args, stream):
           flush=True)
     if st != nexus.OK:
         raise SystemExit(1)
+
+
+def _qkv_measure(wl, stream, peaks, peak_kind, with_oracle, warmup=3, reps=10):
+    """Fresh Q, K, V of re-decoded tokens (one layer per launch), timed apart
+    from the step: all 32768 tokens of the re-prefill (R = 100 %, Sec. III-C)
+    and the 64-token suffix. Inputs exceed L2 (x alone is 335 MB)."""
+    import torch
+
+    from paper_2608_20397_gb300.workloads import HIDDEN, qkv_weights, randn_bf16
+    nexus = wl.nexus
+    dev = wl.kp.device
+    n_heads = HQ + 2 * HKV
+    w, b = qkv_weights(n_heads, HIDDEN, 1001, dev)
+    x = randn_bf16((wl.n_past, HIDDEN), 1000, dev)
+    q = torch.empty((wl.n_past, HQ, D), dtype=torch.bfloat16, device=dev)
+    cases = {"reprefill": (wl.n_past, wl.n_past, 0), "suffix": (wl.T, wl.R_split, 1)}
+    out = {"kernel": "qkv_kernel", "hidden": HIDDEN, "heads": f"{HQ} q + {HKV} k + {HKV} v"}
+    for name, (kv, n, row) in cases.items():
+        def one(l):
+            nexus.suffix_qkv(wl.cache, wl.d_pt, 2, wl.max_pages, [kv], [n], x[:n], w, b, q[:n],
+                             layer=l % wl.L, n_q_heads=HQ, rows=[row], stream=stream)
+        for i in range(warmup):
+            one(i)
+        a = torch.cuda.Event(enable_timing=True)
+        e = torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for i in range(reps):
+            one(i)
+        e.record(stream)
+        torch.cuda.synchronize()
+        ms = a.elapsed_time(e) / reps
+        flops = 2.0 * n * HIDDEN * n_heads * D
+        out[name] = {"tokens": n, "ms_per_launch": ms, "tflops": flops / (ms * 1e-3) / 1e12}
+    st = nexus.device_status(stream)
+    if st != nexus.OK:
+        raise RuntimeError(f"device status after the Q/K/V timing: {nexus.status_string(st)}")
+    achieved = out["reprefill"]["tflops"]
+    out["roofline"] = {"bound": "tensor", "kernel": "qkv_kernel (32768 tokens, one layer)",
+                       "achieved": achieved, "peak": peaks["bf16_tflops"], "unit": "TFLOP/s",
+                       "frac": achieved / peaks["bf16_tflops"],
+                       "peak_kind": f"bf16 burst (timed alone), {peak_kind}",
+                       "traffic": _profiled_traffic("qkv_kernel")}
+    if with_oracle:
+        import oracle
+        n = 64
+        xs = x[:n].float().cpu().double().numpy()
+        wf = w.float().cpu().double().numpy()
+        bf = b.double().cpu().numpy()
+        t0 = time.perf_counter()
+        oracle.qkv_recompute(xs, wf, bf, np.arange(n), HQ, HKV)
+        dt = time.perf_counter() - t0
+        out["cpu_baseline"] = {"value": 2.0 * n * HIDDEN * n_heads * D / dt / 1e12,
+                               "unit": "TFLOP/s", "cores": cpu_cores(), "kind": "oracle",
+                               "sample": f"fp64 NumPy oracle: {n} tokens x {HIDDEN} hidden -> "
+                                         f"{n_heads * D} features, with RoPE", "seconds": dt}
+    return out
 
 
 def _profiled_traffic(kernel: str):

@@ -136,7 +136,9 @@ struct QkvLaunch {
   int32_t n_tok;            // packed tokens (sum of q_len)
   int32_t k_blocks;         // ceil(hidden / 64)
   int32_t n_tiles;          // 256-feature tiles: ceil(n_heads / 2)
-  int32_t total_tiles;      // ceil(n_tok / 128) * n_tiles
+  int32_t m_tiles;          // 128-token tiles: ceil(n_tok / 128)
+  int32_t group_m;          // token tiles per raster band
+  int32_t total_tiles;      // m_tiles * n_tiles
   int32_t n_seqs;
   float inv_freq_hi[kHeadDim / 2];   // theta_i / pi = hi + lo
   float inv_freq_lo[kHeadDim / 2];

@@ -611,6 +611,11 @@ nexus_status nexus_suffix_qkv(const nexus_kv_cache* cache, const int32_t* d_page
   p->n_tok = static_cast<int32_t>(n_tok);
   p->k_blocks = (hidden + 63) / 64;
   p->n_tiles = static_cast<int32_t>(n_tiles);
+  p->m_tiles = static_cast<int32_t>((n_tok + 127) / 128);
+  // A band of token tiles and the weight tiles it meets stay in L2: up to 18
+  // token tiles (1.25 MiB of rows each at hidden 5120) and, across 152 SMs,
+  // about 8 weight tiles (2.5 MiB each) in flight.
+  p->group_m = std::min<int32_t>(p->m_tiles, 18);
   p->total_tiles = static_cast<int32_t>(total);
   p->n_seqs = n_seqs;
   double inv[kHeadDim / 2];

@@ -4,8 +4,10 @@
 // into the token's slot of the paged cache (either V layout, Sec. V-B).
 //
 // Persistent CTAs, one per SM, walk output tiles of 128 tokens x 256 features
-// (two heads), the feature tile fastest so that the CTAs in flight share the
-// weight tiles in L2:
+// (two heads) in bands of group_m token tiles, the token tile fastest inside a
+// band: the tiles in flight at any time share a few weight tiles and the
+// band's token rows, which stay in L2, so DRAM sees each weight tile once per
+// band rather than once per wave:
 //   warp 0     TMA producer: X and W tiles of 64 hidden features per stage,
 //              128-byte swizzle, 4-stage ring (48 KiB a stage)
 //   warp 1     tcgen05.mma issuer (one lane): 128x256x16 bf16 products into
@@ -78,6 +80,16 @@ __device__ __forceinline__ void store_col32(uint16_t* dst, const float (&f)[32])
   for (int i = 0; i < 32; ++i) dst[i * kPageSize] = __bfloat16_as_ushort(__float2bfloat16_rn(f[i]));
 }
 
+__device__ __forceinline__ void tile_coords(const QkvLaunch& p, int t, int& mt, int& nt) {
+  const int per_band = p.group_m * p.n_tiles;
+  const int band = t / per_band;
+  const int first = band * p.group_m;
+  const int gm = min(p.group_m, p.m_tiles - first);
+  const int local = t - band * per_band;
+  mt = first + local % gm;
+  nt = local / gm;
+}
+
 __global__ void __launch_bounds__(kThreads, 1)
 qkv_kernel(const __grid_constant__ QkvLaunch p, const __grid_constant__ QkvMaps maps) {
   extern __shared__ uint8_t smem_raw[];
@@ -124,7 +136,8 @@ qkv_kernel(const __grid_constant__ QkvLaunch p, const __grid_constant__ QkvMaps 
       int it = 0;
       bool ok = true;
       for (int t = blockIdx.x; t < p.total_tiles && ok; t += gridDim.x) {
-        const int mt = t / p.n_tiles, nt = t % p.n_tiles;
+        int mt, nt;
+        tile_coords(p, t, mt, nt);
         for (int kb = 0; kb < p.k_blocks; ++kb, ++it) {
           const int st = it % kStages;
           if (it >= kStages) {
@@ -186,7 +199,8 @@ qkv_kernel(const __grid_constant__ QkvLaunch p, const __grid_constant__ QkvMaps 
     const int64_t page_elems = (int64_t)p.n_kv_heads * kPageSize * kHeadDim;
     int acc_it = 0;
     for (int t = blockIdx.x; t < p.total_tiles; t += gridDim.x, ++acc_it) {
-      const int mt = t / p.n_tiles, nt = t % p.n_tiles;
+      int mt, nt;
+      tile_coords(p, t, mt, nt);
       const int buf = acc_it & 1;
       bool ok = mbar_wait(bar(B_AFULL + buf), (acc_it >> 1) & 1, kBudgetNs, abort, gabort);
       ok = __all_sync(0xffffffffu, ok);
