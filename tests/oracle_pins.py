@@ -403,3 +403,89 @@ def pin_qkv_recompute(qkv_recompute, rope_rotate):
     assert np.max(np.abs(qp - rope_rotate(q0, pos[:, None]))) < 1e-11
     assert np.max(np.abs(kp - rope_rotate(k0, pos[:, None]))) < 1e-11
     assert np.array_equal(vp, v0)
+
+
+def pin_common_prefix_len(common_prefix_len):
+    """Exact-token common prefix (Sec. V-D): the library's os.path.commonprefix
+    on lists, the whole sequence against itself or an extension, the index of
+    the first changed token, symmetry and the empty sequence."""
+    import os.path
+    r = _rs(23)
+    for _ in range(200):
+        n = int(r.integers(0, 40))
+        a = [int(t) for t in r.integers(0, 5, n)]
+        b = a[: int(r.integers(0, n + 1))] + [int(t) for t in r.integers(0, 5, int(r.integers(0, 9)))]
+        want = len(os.path.commonprefix([a, b]))
+        assert common_prefix_len(a, b) == want == common_prefix_len(b, a)
+        assert common_prefix_len(a, a) == len(a)
+        assert common_prefix_len(a, a + [7, 8]) == len(a)
+        if n:
+            i = int(r.integers(0, n))
+            c = list(a); c[i] = c[i] + 11
+            assert common_prefix_len(a, c) == i
+    assert common_prefix_len([], [1, 2]) == 0
+
+
+def pin_warm_match(warm_match, common_prefix_len):
+    """Best slot = the longest exact-token prefix, ties to the latest use, a
+    miss when no slot shares the first token; empty slots are skipped."""
+    r = _rs(24)
+    for _ in range(300):
+        n_slots = int(r.integers(1, 7))
+        base = [int(t) for t in r.integers(0, 3, 12)]
+        slots = []
+        for _s in range(n_slots):
+            if r.random() < 0.2:
+                slots.append(None)
+                continue
+            cut = int(r.integers(0, 13))
+            slots.append(base[:cut] + [int(t) for t in r.integers(0, 3, int(r.integers(0, 6)))])
+        uses = [int(u) for u in r.permutation(n_slots) + 1]
+        q = base[: int(r.integers(0, 13))] + [int(t) for t in r.integers(0, 3, 3)]
+        s, m = warm_match(slots, uses, q)
+        lens = [common_prefix_len(t, q) if t is not None else 0 for t in slots]
+        assert m == max(lens + [0])
+        if m == 0:
+            assert s == -1
+        else:
+            ties = [i for i in range(n_slots) if slots[i] is not None and lens[i] == m]
+            assert s == max(ties, key=lambda i: uses[i])
+    # a hand-made tie: both slots share 3 tokens, slot 0 used later
+    assert warm_match([[1, 2, 3, 9], [1, 2, 3, 8]], [5, 4], [1, 2, 3, 7]) == (0, 3)
+    assert warm_match([[1, 2, 3, 9], [1, 2, 3, 8]], [4, 5], [1, 2, 3, 7]) == (1, 3)
+    assert warm_match([[4, 5], None], [1, 0], [5, 4]) == (-1, 0)
+
+
+def pin_warm_arena(WarmArenaModel):
+    """The arena's decisions on hand-made scenarios: reuse of a stored prefix
+    with its exact rows, LRU eviction, in-place extension of a slot, a stored
+    prefix of a slot refreshes it, truncation at max_tokens, and forks are
+    copies that later stores do not change."""
+    def rows(tokens):   # K = V = one row per token holding the token value
+        a = np.asarray(tokens, dtype=np.float64).reshape(1, -1, 1, 1)
+        return a, -a
+    A = list(range(100))
+    arena = WarmArenaModel(n_slots=3, max_tokens=120)
+    sa = arena.store(A, *rows(A))
+    assert sa == 0 and arena.match(A) == (0, 100)
+    assert arena.match(A[:50] + [999]) == (0, 50)
+    assert arena.match([999] + A) == (-1, 0)
+    k, v = arena.fork(0, 37)
+    assert np.array_equal(k, rows(A)[0][:, :37]) and np.array_equal(v, rows(A)[1][:, :37])
+    B, C, D = [1000 + t for t in A], [2000 + t for t in A], [3000 + t for t in A]
+    assert arena.store(B, *rows(B)) == 1 and arena.store(C, *rows(C)) == 2
+    arena.fork(0, 10)                        # A is now used after B and C
+    assert arena.store(D, *rows(D)) == 1     # B, the least recently used, is evicted
+    assert arena.match(B)[0] == -1 and arena.match(A) == (0, 100)
+    A2 = A + [500, 501]
+    assert arena.store(A2, *rows(A2)) == 0   # an extension replaces its prefix's slot
+    assert arena.match(A2) == (0, 102)
+    assert arena.store(A[:60], *rows(A[:60])) == 0 and arena.match(A2) == (0, 102)
+    E = [4000 + t for t in range(200)]
+    se = arena.store(E, *rows(E))
+    assert arena.match(E) == (se, 120)       # only the first max_tokens tokens are kept
+    k_before, _ = arena.fork(se, 120)
+    F = [5000 + t for t in range(5)]
+    arena.store(F, *rows(F))
+    arena.store([6000], *rows([6000]))
+    assert np.array_equal(k_before, rows(E)[0][:, :120])

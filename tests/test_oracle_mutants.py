@@ -218,3 +218,52 @@ def test_qkv_mutants_caught():
 
     for mut in (transposed_weight, kv_swapped, no_bias, v_rotated):
         assert _fails(P.pin_qkv_recompute, mut, oracle.rope_rotate), mut.__name__
+
+
+def test_arena_mutants_caught():
+    def lcp_counts_mismatch(a, b):
+        n = oracle.common_prefix_len(a, b)
+        return n + 1 if n < min(len(a), len(b)) else n
+
+    assert _fails(P.pin_common_prefix_len, lcp_counts_mismatch)
+
+    def match_ties_to_oldest(slots, uses, q):
+        best, best_len, best_use = -1, 0, None
+        for s, t in enumerate(slots):
+            if t is None:
+                continue
+            n = oracle.common_prefix_len(t, q)
+            if n and (n > best_len or (n == best_len and uses[s] < best_use)):
+                best, best_len, best_use = s, n, uses[s]
+        return best, best_len
+
+    assert _fails(P.pin_warm_match, match_ties_to_oldest, oracle.common_prefix_len)
+
+    class EvictsMostRecent(oracle.WarmArenaModel):
+        """Evicts the most recently used slot when the arena is full."""
+        def store(self, tokens, k, v):
+            toks = [int(t) for t in tokens[: self.max_tokens]]
+            related = any(t is not None and (t[: len(toks)] == toks or toks[: len(t)] == t)
+                          for t in self.tokens)
+            if not related and all(t is not None for t in self.tokens):
+                self.tokens[max(range(self.n_slots), key=lambda i: self.last_use[i])] = None
+            return super().store(tokens, k, v)
+
+    class NoExtension(oracle.WarmArenaModel):
+        """Never replaces a slot whose tokens are a prefix of the stored ones."""
+        def store(self, tokens, k, v):
+            toks = [int(t) for t in tokens[: self.max_tokens]]
+            for s, t in enumerate(self.tokens):
+                if t is not None and len(t) >= len(toks) and t[: len(toks)] == toks:
+                    self._touch(s)
+                    return s
+            empty = [s for s, t in enumerate(self.tokens) if t is None]
+            s = empty[0] if empty else min(range(self.n_slots), key=lambda i: self.last_use[i])
+            self.tokens[s] = toks
+            self.k[s] = np.array(k[:, : len(toks)])
+            self.v[s] = np.array(v[:, : len(toks)])
+            self._touch(s)
+            return s
+
+    for mut in (EvictsMostRecent, NoExtension):
+        assert _fails(P.pin_warm_arena, mut), mut.__name__

@@ -79,3 +79,15 @@ def test_attention_softcap():
 
 def test_qkv_recompute():
     P.pin_qkv_recompute(oracle.qkv_recompute, oracle.rope_rotate)
+
+
+def test_common_prefix_len():
+    P.pin_common_prefix_len(oracle.common_prefix_len)
+
+
+def test_warm_match():
+    P.pin_warm_match(oracle.warm_match, oracle.common_prefix_len)
+
+
+def test_warm_arena():
+    P.pin_warm_arena(oracle.WarmArenaModel)
