@@ -25,7 +25,10 @@
  *                            the depth-adaptive policy of Eq. 2 and the
  *                            splice threshold P (Sec. III-B, Sec. III-C)
  *   nexus_page_pool_*, nexus_plan_splice
- *                            host page allocator and splice planner
+ *                            host page allocator (reference-counted pages,
+ *                            copy-on-write) and splice planner
+ *   nexus_warm_arena_*       the L0 exact-token radix arena of warm prefixes
+ *                            (Sec. V-D)
  *
  * Conventions
  *   - Device buffers are owned by the caller. The library never allocates or
@@ -180,10 +183,77 @@ nexus_status nexus_page_pool_create(int64_t n_pages, const int32_t* order,
 void nexus_page_pool_destroy(nexus_page_pool* pool);
 /* Takes n pages in pool order; NEXUS_ENOMEM (and no change) if fewer are free. */
 nexus_status nexus_page_pool_alloc(nexus_page_pool* pool, int32_t n, int32_t* pages);
-/* Returns pages to the back of the order; NEXUS_ERANGE for an id outside the
- * pool, NEXUS_EINVAL for a page that is already free (nothing is freed then). */
+/* Drops one reference from each page; a page whose last reference goes returns
+ * to the back of the order. NEXUS_ERANGE for an id outside the pool,
+ * NEXUS_EINVAL for a page that is already free or listed twice (nothing
+ * changes then). */
 nexus_status nexus_page_pool_free(nexus_page_pool* pool, int32_t n, const int32_t* pages);
 int64_t nexus_page_pool_available(const nexus_page_pool* pool);
+/* Adds one reference to each page, for a page shared by several page tables
+ * (a warm prefix, Sec. V-D). Each page must be in use and listed once;
+ * NEXUS_EINVAL / NEXUS_ERANGE otherwise (nothing changes). A page goes back to
+ * the pool when nexus_page_pool_free has dropped every reference. */
+nexus_status nexus_page_pool_retain(nexus_page_pool* pool, int32_t n, const int32_t* pages);
+/* References held on a page: 0 when free, -1 for an id outside the pool. */
+int64_t nexus_page_pool_refs(const nexus_page_pool* pool, int32_t page);
+/* Copy-on-write before rows are written in place: every page of
+ * h_pt[first_page, first_page + n) with more than one reference is replaced in
+ * h_pt by a fresh page, the table's reference on the old page is dropped, and
+ * the (old, fresh) pairs are written to src_pages / dst_pages (capacity pairs)
+ * for nexus_copy_pages, which must run before the rows are written.
+ * NEXUS_ENOMEM (nothing changes) if the pool or the capacity is too small. */
+nexus_status nexus_page_pool_make_private(nexus_page_pool* pool, int32_t* h_pt,
+                                          int32_t first_page, int32_t n, int32_t* src_pages,
+                                          int32_t* dst_pages, int32_t capacity,
+                                          int32_t* n_copies);
+
+/* ---------------------------------------------------------- L0 warm arena */
+/* The L0 exact-token radix arena (Sec. V-D): n_slots (1..32) sequence slots of
+ * up to max_tokens tokens. A new request looks up the slot sharing the longest
+ * exact-token prefix with it and starts from that prefix's KV instead of
+ * recomputing it. A slot holds its sequence's tokens and one reference on each
+ * cache page of its rows (no copy); a sequence forked from a slot shares the
+ * pages that hold only prefix rows and gets a private copy of the page it will
+ * go on writing, so reusing m warm tokens costs at most one page copy.
+ * Rule for callers: rows [0, n) of a stored sequence must keep their bits while
+ * a slot holds them; before writing any of them in place (re-rotation, Q/K/V
+ * recompute of a suffix), make their pages private
+ * (nexus_page_pool_make_private). Writing rows past n is free: slots never read
+ * them. All memory is reserved by create; match, fork and store allocate
+ * nothing. An arena is not thread-safe: serialise calls on one arena. */
+typedef struct nexus_warm_arena nexus_warm_arena;
+nexus_status nexus_warm_arena_create(int32_t n_slots, int32_t max_tokens,
+                                     nexus_warm_arena** out);
+/* Drops the slots' page references into `pool` (nullable) and frees the arena. */
+void nexus_warm_arena_destroy(nexus_warm_arena* arena, nexus_page_pool* pool);
+/* The slot sharing the longest exact-token prefix with tokens[0, n): *slot and
+ * *prefix (its length); equal prefixes go to the most recently used slot;
+ * *slot = -1, *prefix = 0 when no slot shares the first token. Changes no slot. */
+nexus_status nexus_warm_arena_match(nexus_warm_arena* arena, const int32_t* tokens, int32_t n,
+                                    int32_t* slot, int32_t* prefix);
+/* Starts a sequence from the first m tokens of `slot` (m <= its length):
+ * writes h_new_pt[0, ceil(m / 16)). Pages holding only rows < m are shared
+ * (one more reference each); when m is not a multiple of 16 the page holding
+ * row m - 1 is copied to a fresh page from `pool`, returned as one pair in
+ * copy_src[0] -> copy_dst[0] (*n_copies = 1) for nexus_copy_pages. The new
+ * sequence then writes its rows m.. itself. Counts as a use of the slot. */
+nexus_status nexus_warm_arena_fork(nexus_warm_arena* arena, nexus_page_pool* pool, int32_t slot,
+                                   int32_t m, int32_t* h_new_pt, int32_t max_pages,
+                                   int32_t* copy_src, int32_t* copy_dst, int32_t* n_copies);
+/* Enters a sequence of n tokens whose rows live in the pages h_pt[0, ceil(n' /
+ * 16)), n' = min(n, max_tokens). If a slot already holds a sequence starting
+ * with these n' tokens, only its use is refreshed. Otherwise the sequence
+ * replaces the longest slot that holds a prefix of it, else the lowest empty
+ * slot, else the least recently used one; that slot takes a reference on each
+ * of the pages and drops those of the sequence it held. *slot_out (nullable)
+ * receives the slot. */
+nexus_status nexus_warm_arena_store(nexus_warm_arena* arena, nexus_page_pool* pool,
+                                    const int32_t* tokens, int32_t n, const int32_t* h_pt,
+                                    int32_t* slot_out);
+/* A slot's token count (0 = empty) and, when h_pages is given, its pages
+ * (capacity >= ceil(count / 16), else NEXUS_ENOMEM). */
+nexus_status nexus_warm_arena_slot(const nexus_warm_arena* arena, int32_t slot, int32_t* n_tokens,
+                                   int32_t* h_pages, int32_t capacity);
 
 /* --------------------------------------------------------------- planner */
 /* Plans the insertion of blocks into one sequence of length n_past whose page

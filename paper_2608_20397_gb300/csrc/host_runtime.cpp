@@ -2,8 +2,8 @@
 // Sec. III-C), the fail-closed splice gate (Sec. III-B), the page pool
 // (Sec. V-C analogue) and the splice planner (Sec. III-B / Sec. V-A).
 #include <algorithm>
+#include <cstdint>
 #include <cstring>
-#include <deque>
 #include <mutex>
 #include <new>
 #include <numeric>
@@ -51,16 +51,52 @@ int32_t ceil_fraction(int32_t S, int64_t num, int64_t den) {
 }  // namespace
 
 // ------------------------------------------------------------------ pool
-// Page ids are handed out in the order of `order`; freed pages go to the
-// back. The mutex sits on its own 128-byte line, away from the data the
-// allocating threads read, so contended locking does not false-share.
+// Page ids are handed out in the order of `order`; a page whose last reference
+// is dropped goes to the back. Pages may be shared by several page tables (a
+// warm prefix, Sec. V-D), so each carries a reference count. All storage is
+// reserved at creation: alloc, retain and free never allocate. The mutex sits
+// on its own 128-byte line, away from the data the allocating threads read, so
+// contended locking does not false-share.
 struct alignas(128) nexus_page_pool {
   alignas(128) std::mutex mu;
   alignas(128) int64_t n_pages = 0;
-  std::deque<int32_t> free_order;
-  std::vector<uint8_t> in_use;
+  std::vector<int32_t> ring;    // free pages in hand-out order: ring[head .. head + n_free)
+  int64_t head = 0;
+  int64_t n_free = 0;
+  std::vector<uint32_t> refs;   // references per page; 0 = free
+  std::vector<uint32_t> mark;   // duplicate check of one request (epoch stamps)
+  uint32_t epoch = 0;
 };
 static_assert(alignof(nexus_page_pool) % 128 == 0, "page pool must be cache-line aligned");
+
+namespace {
+
+void ring_push(nexus_page_pool* p, int32_t pg) {
+  p->ring[static_cast<size_t>((p->head + p->n_free) % p->n_pages)] = pg;
+  ++p->n_free;
+}
+
+int32_t ring_pop(nexus_page_pool* p) {
+  const int32_t pg = p->ring[static_cast<size_t>(p->head)];
+  p->head = (p->head + 1) % p->n_pages;
+  --p->n_free;
+  return pg;
+}
+
+// Stamps pages[0, n) for one request; false if a page repeats. Caller holds mu.
+bool distinct(nexus_page_pool* p, int32_t n, const int32_t* pages) {
+  if (++p->epoch == 0) {
+    std::fill(p->mark.begin(), p->mark.end(), 0u);
+    p->epoch = 1;
+  }
+  for (int32_t i = 0; i < n; ++i) {
+    if (p->mark[pages[i]] == p->epoch) return false;
+    p->mark[pages[i]] = p->epoch;
+  }
+  return true;
+}
+
+}  // namespace
 
 extern "C" {
 
@@ -114,18 +150,21 @@ nexus_status nexus_page_pool_create(int64_t n_pages, const int32_t* order, nexus
   nexus_page_pool* pool = new (std::nothrow) nexus_page_pool();
   if (!pool) return NEXUS_ENOMEM;
   pool->n_pages = n_pages;
-  pool->in_use.assign(static_cast<size_t>(n_pages), 0);
+  pool->refs.assign(static_cast<size_t>(n_pages), 0u);
+  pool->mark.assign(static_cast<size_t>(n_pages), 0u);
+  pool->ring.assign(static_cast<size_t>(n_pages), 0);
   if (order) {
-    std::vector<uint8_t> seen(static_cast<size_t>(n_pages), 0);
     for (int64_t i = 0; i < n_pages; ++i) {
       const int32_t pg = order[i];
-      if (pg < 0 || pg >= n_pages || seen[pg]) { delete pool; return NEXUS_EINVAL; }
-      seen[pg] = 1;
-      pool->free_order.push_back(pg);
+      if (pg < 0 || pg >= n_pages || pool->mark[pg]) { delete pool; return NEXUS_EINVAL; }
+      pool->mark[pg] = 1;
+      pool->ring[i] = pg;
     }
+    std::fill(pool->mark.begin(), pool->mark.end(), 0u);
   } else {
-    for (int64_t i = 0; i < n_pages; ++i) pool->free_order.push_back(static_cast<int32_t>(i));
+    for (int64_t i = 0; i < n_pages; ++i) pool->ring[i] = static_cast<int32_t>(i);
   }
+  pool->n_free = n_pages;
   *out = pool;
   return NEXUS_OK;
 }
@@ -135,11 +174,10 @@ void nexus_page_pool_destroy(nexus_page_pool* pool) { delete pool; }
 nexus_status nexus_page_pool_alloc(nexus_page_pool* pool, int32_t n, int32_t* pages) {
   if (!pool || n < 0 || (n > 0 && !pages)) return NEXUS_EINVAL;
   std::lock_guard<std::mutex> lock(pool->mu);
-  if (static_cast<int64_t>(pool->free_order.size()) < n) return NEXUS_ENOMEM;
+  if (pool->n_free < n) return NEXUS_ENOMEM;
   for (int32_t i = 0; i < n; ++i) {
-    const int32_t pg = pool->free_order.front();
-    pool->free_order.pop_front();
-    pool->in_use[pg] = 1;
+    const int32_t pg = ring_pop(pool);
+    pool->refs[pg] = 1;
     pages[i] = pg;
   }
   return NEXUS_OK;
@@ -148,26 +186,70 @@ nexus_status nexus_page_pool_alloc(nexus_page_pool* pool, int32_t n, int32_t* pa
 nexus_status nexus_page_pool_free(nexus_page_pool* pool, int32_t n, const int32_t* pages) {
   if (!pool || n < 0 || (n > 0 && !pages)) return NEXUS_EINVAL;
   std::lock_guard<std::mutex> lock(pool->mu);
-  std::vector<int32_t> seen;
   for (int32_t i = 0; i < n; ++i) {
     if (pages[i] < 0 || pages[i] >= pool->n_pages) return NEXUS_ERANGE;
-    if (!pool->in_use[pages[i]]) return NEXUS_EINVAL;
+    if (pool->refs[pages[i]] == 0) return NEXUS_EINVAL;
   }
-  // reject duplicates inside the request as a double free
-  seen.assign(pages, pages + n);
-  std::sort(seen.begin(), seen.end());
-  if (std::adjacent_find(seen.begin(), seen.end()) != seen.end()) return NEXUS_EINVAL;
-  for (int32_t i = 0; i < n; ++i) {
-    pool->in_use[pages[i]] = 0;
-    pool->free_order.push_back(pages[i]);
-  }
+  if (!distinct(pool, n, pages)) return NEXUS_EINVAL;   // a page listed twice
+  for (int32_t i = 0; i < n; ++i)
+    if (--pool->refs[pages[i]] == 0) ring_push(pool, pages[i]);
   return NEXUS_OK;
+}
+
+nexus_status nexus_page_pool_retain(nexus_page_pool* pool, int32_t n, const int32_t* pages) {
+  if (!pool || n < 0 || (n > 0 && !pages)) return NEXUS_EINVAL;
+  std::lock_guard<std::mutex> lock(pool->mu);
+  for (int32_t i = 0; i < n; ++i) {
+    if (pages[i] < 0 || pages[i] >= pool->n_pages) return NEXUS_ERANGE;
+    if (pool->refs[pages[i]] == 0 || pool->refs[pages[i]] == UINT32_MAX) return NEXUS_EINVAL;
+  }
+  if (!distinct(pool, n, pages)) return NEXUS_EINVAL;
+  for (int32_t i = 0; i < n; ++i) ++pool->refs[pages[i]];
+  return NEXUS_OK;
+}
+
+int64_t nexus_page_pool_refs(const nexus_page_pool* pool, int32_t page) {
+  if (!pool || page < 0 || page >= pool->n_pages) return -1;
+  std::lock_guard<std::mutex> lock(const_cast<nexus_page_pool*>(pool)->mu);
+  return pool->refs[page];
 }
 
 int64_t nexus_page_pool_available(const nexus_page_pool* pool) {
   if (!pool) return -1;
   std::lock_guard<std::mutex> lock(const_cast<nexus_page_pool*>(pool)->mu);
-  return static_cast<int64_t>(pool->free_order.size());
+  return pool->n_free;
+}
+
+nexus_status nexus_page_pool_make_private(nexus_page_pool* pool, int32_t* h_pt, int32_t first_page,
+                                          int32_t n, int32_t* src_pages, int32_t* dst_pages,
+                                          int32_t capacity, int32_t* n_copies) {
+  if (!pool || !h_pt || first_page < 0 || n < 0 || !n_copies || capacity < 0) return NEXUS_EINVAL;
+  *n_copies = 0;
+  std::lock_guard<std::mutex> lock(pool->mu);
+  int32_t shared = 0;
+  for (int32_t i = first_page; i < first_page + n; ++i) {
+    const int32_t pg = h_pt[i];
+    if (pg < 0 || pg >= pool->n_pages) return NEXUS_ERANGE;
+    if (pool->refs[pg] == 0) return NEXUS_EINVAL;
+    if (pool->refs[pg] > 1) ++shared;
+  }
+  if (shared > capacity || (shared > 0 && (!src_pages || !dst_pages))) return NEXUS_ENOMEM;
+  if (shared > pool->n_free) return NEXUS_ENOMEM;
+  if (!distinct(pool, n, h_pt + first_page)) return NEXUS_EINVAL;   // one page twice in a table
+  int32_t k = 0;
+  for (int32_t i = first_page; i < first_page + n; ++i) {
+    const int32_t pg = h_pt[i];
+    if (pool->refs[pg] <= 1) continue;
+    const int32_t fresh = ring_pop(pool);
+    pool->refs[fresh] = 1;
+    --pool->refs[pg];   // still referenced elsewhere: stays in use
+    src_pages[k] = pg;
+    dst_pages[k] = fresh;
+    h_pt[i] = fresh;
+    ++k;
+  }
+  *n_copies = k;
+  return NEXUS_OK;
 }
 
 nexus_status nexus_plan_splice(nexus_page_pool* pool, const int32_t* h_old_pt, int32_t n_past,

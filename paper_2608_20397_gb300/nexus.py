@@ -84,6 +84,17 @@ _SIGS = {
     "nexus_page_pool_alloc": (c_int32, [c_void_p, c_int32, _i32p]),
     "nexus_page_pool_free": (c_int32, [c_void_p, c_int32, _i32p]),
     "nexus_page_pool_available": (c_int64, [c_void_p]),
+    "nexus_page_pool_retain": (c_int32, [c_void_p, c_int32, _i32p]),
+    "nexus_page_pool_refs": (c_int64, [c_void_p, c_int32]),
+    "nexus_page_pool_make_private": (c_int32, [c_void_p, _i32p, c_int32, c_int32, _i32p, _i32p,
+                                               c_int32, _i32p]),
+    "nexus_warm_arena_create": (c_int32, [c_int32, c_int32, POINTER(c_void_p)]),
+    "nexus_warm_arena_destroy": (None, [c_void_p, c_void_p]),
+    "nexus_warm_arena_match": (c_int32, [c_void_p, _i32p, c_int32, _i32p, _i32p]),
+    "nexus_warm_arena_fork": (c_int32, [c_void_p, c_void_p, c_int32, c_int32, _i32p, c_int32,
+                                        _i32p, _i32p, _i32p]),
+    "nexus_warm_arena_store": (c_int32, [c_void_p, c_void_p, _i32p, c_int32, _i32p, _i32p]),
+    "nexus_warm_arena_slot": (c_int32, [c_void_p, c_int32, _i32p, _i32p, c_int32]),
     "nexus_plan_splice": (c_int32, [c_void_p, _i32p, c_int32, c_int32, POINTER(Block), c_int32,
                                     POINTER(Insert), c_int32, c_int32, c_int32, _i32p,
                                     POINTER(Segment), c_int32, _i32p, _i32p, _i32p]),
@@ -234,6 +245,26 @@ class PagePool:
 
     def available(self) -> int:
         return int(lib().nexus_page_pool_available(self._h))
+
+    def retain(self, pages) -> None:
+        buf = _i32(pages)
+        _check("nexus_page_pool_retain", lib().nexus_page_pool_retain(self._h, len(buf[1]), buf[0]))
+
+    def refs(self, page: int) -> int:
+        return int(lib().nexus_page_pool_refs(self._h, int(page)))
+
+    def make_private(self, pt: np.ndarray, first_page: int, n: int):
+        """Copy-on-write of pt[first_page, first_page + n) in place (pt: int32
+        array); returns the (old, fresh) page pairs to copy before writing."""
+        assert pt.dtype == np.int32 and pt.flags.c_contiguous
+        cap = max(int(n), 1)
+        src = np.zeros(cap, np.int32)
+        dst = np.zeros(cap, np.int32)
+        k = c_int32()
+        _check("nexus_page_pool_make_private", lib().nexus_page_pool_make_private(
+            self._h, pt.ctypes.data_as(_i32p), int(first_page), int(n),
+            src.ctypes.data_as(_i32p), dst.ctypes.data_as(_i32p), cap, ctypes.byref(k)))
+        return src[:k.value].copy(), dst[:k.value].copy()
 
     def close(self):
         if self._h:
@@ -418,3 +449,62 @@ def suffix_qkv(cache: KvCache, d_page_tables, n_rows: int, max_pages: int, kv_le
         int(max_pages), len(kv[1]), rw[0] if rw else None, kv[0], ql[0], _ptr(x),
         int(hidden if hidden is not None else x.shape[-1]), _ptr(w_qkv), _ptr(b_qkv), int(n_q_heads),
         int(layer), _ptr(q_out), _stream(stream)))
+
+
+# ------------------------------------------------------------ warm arena
+class WarmArena:
+    """The L0 exact-token radix arena of warm prefixes (see nexus.h)."""
+
+    def __init__(self, n_slots: int = 32, max_tokens: int = 1 << 16):
+        h = c_void_p()
+        _check("nexus_warm_arena_create",
+               lib().nexus_warm_arena_create(int(n_slots), int(max_tokens), ctypes.byref(h)))
+        self._h = h
+        self.n_slots = int(n_slots)
+        self.max_tokens = int(max_tokens)
+
+    def match(self, tokens):
+        buf = _i32(tokens)
+        slot, pre = c_int32(), c_int32()
+        _check("nexus_warm_arena_match", lib().nexus_warm_arena_match(
+            self._h, buf[0], len(buf[1]), ctypes.byref(slot), ctypes.byref(pre)))
+        return slot.value, pre.value
+
+    def fork(self, pool: PagePool, slot: int, m: int, max_pages: int):
+        """Page table prefix (int32 [ceil(m / 16)]) of a sequence started from
+        the first m tokens of `slot`, and the page copies to run first."""
+        pt = np.full(max(int(max_pages), 1), -1, np.int32)
+        src = np.zeros(1, np.int32)
+        dst = np.zeros(1, np.int32)
+        k = c_int32()
+        _check("nexus_warm_arena_fork", lib().nexus_warm_arena_fork(
+            self._h, pool.handle, int(slot), int(m), pt.ctypes.data_as(_i32p), int(max_pages),
+            src.ctypes.data_as(_i32p), dst.ctypes.data_as(_i32p), ctypes.byref(k)))
+        return pt[: -(-int(m) // 16)].copy(), src[:k.value].copy(), dst[:k.value].copy()
+
+    def store(self, pool: PagePool, tokens, pt) -> int:
+        tb = _i32(tokens)
+        pb = _i32(pt)
+        slot = c_int32()
+        _check("nexus_warm_arena_store", lib().nexus_warm_arena_store(
+            self._h, pool.handle, tb[0], len(tb[1]), pb[0], ctypes.byref(slot)))
+        return slot.value
+
+    def slot(self, slot: int):
+        """(token count, pages) of a slot."""
+        n = c_int32()
+        pages = np.zeros(-(-self.max_tokens // 16), np.int32)
+        _check("nexus_warm_arena_slot", lib().nexus_warm_arena_slot(
+            self._h, int(slot), ctypes.byref(n), pages.ctypes.data_as(_i32p), len(pages)))
+        return n.value, pages[: -(-n.value // 16)].copy()
+
+    def close(self, pool: Optional[PagePool] = None):
+        if self._h:
+            lib().nexus_warm_arena_destroy(self._h, pool.handle if pool is not None else None)
+            self._h = c_void_p()
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
