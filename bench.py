@@ -16,7 +16,8 @@ The printed metric is attention TFLOP/s over the whole step (algorithmic,
 causal-visible flops 4 d Hq (R (T - R) + R (R + 1) / 2) per layer), with the
 splice GB/s (8192 algorithmic bytes per moved token-layer) beside it. The fresh
 Q/K/V of re-decoded tokens (projection + RoPE + cache write) is timed apart from
-the step under "qkv_recompute" (2 x 5120 x 7168 flops per token).
+the step under "qkv_recompute" (2 x 5120 x 7168 flops per token), and the L0
+warm arena (prefix match, fork, one boundary-page copy) under "l0_arena".
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
 
@@ -302,6 +303,8 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-qkv", action="store_true",
                     help="skip the separate timing of the suffix Q/K/V recompute")
+    ap.add_argument("--no-arena", action="store_true",
+                    help="skip the separate timing of the L0 warm arena")
     ap.add_argument("--layers", type=int, default=48, help="layers of the workload (48 = c5)")
     ap.add_argument("--profile", choices=["reprefill", "reprefill-softcap", "splice", "suffix",
                                           "qkv"],
@@ -400,6 +403,11 @@ def main():
         qkv = _qkv_measure(wl, stream, peaks, peak_kind,
                            with_oracle=rank == 0 and world == 1 and not args.no_cpu_baseline)
 
+    arena = None
+    if not args.no_arena:
+        arena = _arena_measure(wl, stream, peaks, peak_kind,
+                               with_oracle=rank == 0 and world == 1 and not args.no_cpu_baseline)
+
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         f64 = lambda t: t.float().cpu().double().numpy()
@@ -424,7 +432,7 @@ def main():
             "splice_gbs": splice_gbs, "splice_ms": splice_ms, "reprefill_ms": pre_ms,
             "suffix_ms": suf_ms, "suffix_tflops": suf_tflops,
             "roofline": roofline, "roofline_splice": roofline_splice,
-            "e2e": e2e, "cpu_baseline": cpu, "clocks": clocks, "qkv_recompute": qkv,
+            "e2e": e2e, "cpu_baseline": cpu, "clocks": clocks, "qkv_recompute": qkv, "l0_arena": arena,
             "gpu_launches": wl.launches_per_step * args.steps,
         }
         print(json.dumps(line), flush=True)
@@ -558,6 +566,147 @@ def _qkv_measure(wl, stream, peaks, peak_kind, with_oracle, warmup=3, reps=10):
                                "unit": "TFLOP/s", "cores": cpu_cores(), "kind": "oracle",
                                "sample": f"fp64 NumPy oracle: {n} tokens x {HIDDEN} hidden -> "
                                          f"{n_heads * D} features, with RoPE", "seconds": dt}
+    return out
+
+
+def _arena_measure(wl, stream, peaks, peak_kind, with_oracle, n_slots=32, system_len=8192,
+                   tail_len=1024, n_requests=200):
+    """The L0 warm arena (Sec. V-D), timed apart from the step on a cache of the
+    c5 model shape (48 layers, 8 KV heads): 32 slots holding a shared
+    8192-token system prompt plus a 1024-token tail each; every request shares
+    the prompt and part of one tail, so it forks 8192 + k warm tokens (k random)
+    and copies one boundary page of all 48 layers. Also the warm-hit rate of
+    the arena on a seeded stream of agent requests (context: it depends wholly on
+    the stream)."""
+    import torch
+
+    from paper_2608_20397_gb300.workloads import agent_requests
+    nexus = wl.nexus
+    dev = wl.kp.device
+    L = wl.L
+    r = np.random.default_rng(77)
+    sys_pages = system_len // PAGE
+    tail_pages = tail_len // PAGE
+    n_pages = sys_pages + n_slots * tail_pages + 64
+    kp = torch.zeros((L, n_pages, HKV, PAGE, D), dtype=torch.bfloat16, device=dev)
+    vp = torch.zeros_like(kp)
+    cache = nexus.kv_cache(kp, vp, n_pages, L, HKV)
+    pool = nexus.PagePool(n_pages)
+    arena = nexus.WarmArena(n_slots, system_len + tail_len)
+    system = [int(t) for t in r.integers(0, 32000, system_len)]
+    sys_pt = pool.alloc(sys_pages)
+    tails = []
+    for s in range(n_slots):
+        tail = [int(t) for t in r.integers(0, 32000, tail_len)]
+        tails.append(tail)
+        pt = np.concatenate([sys_pt, pool.alloc(tail_pages)]).astype(np.int32)
+        pool.retain(sys_pt)
+        arena.store(pool, system + tail, pt)
+        pool.free(pt)
+    pool.free(sys_pt)            # the slots alone hold the pages now
+    reqs = []
+    for i in range(n_requests + 10):
+        j = int(r.integers(0, n_slots))
+        k = int(r.integers(1, tail_len))
+        q = system + tails[j][:k] + [int(t) for t in r.integers(32000, 33000, 64)]
+        reqs.append((np.asarray(q, dtype=np.int32), system_len + k))
+    # one request at a time, as a server sees it: match, fork, boundary copy, done
+    t_match, t_fork, t_e2e = [], [], []
+    for i, (q, m_want) in enumerate(reqs):
+        stream.synchronize()
+        t0 = time.perf_counter()
+        slot, m = arena.match(q)
+        t1 = time.perf_counter()
+        pt, src, dst = arena.fork(pool, slot, m, -(-len(q) // PAGE))
+        t2 = time.perf_counter()
+        if len(src):
+            nexus.copy_pages(cache, src, dst, 0, L, stream)
+        stream.synchronize()
+        t3 = time.perf_counter()
+        assert m >= m_want
+        pool.free(pt)
+        if i >= 10:
+            t_match.append(t1 - t0)
+            t_fork.append(t2 - t1)
+            t_e2e.append(t3 - t0)
+    # the boundary copies alone: a batch enqueued while the stream is held busy
+    # by a fixed-length sleep, so the events see no host gaps
+    t_copy = []
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
+    for rep in range(5):
+        plans = []
+        for q, _ in reqs[rep * 40:(rep + 1) * 40]:
+            slot, m = arena.match(q)
+            plans.append(arena.fork(pool, slot, m, -(-len(q) // PAGE)))
+        copies = [(src, dst) for _, src, dst in plans if len(src)]
+        torch.cuda._sleep(4_000_000)
+        ev[0].record(stream)
+        for src, dst in copies:
+            nexus.copy_pages(cache, src, dst, 0, L, stream)
+        ev[1].record(stream)
+        ev[1].synchronize()
+        if rep > 0 and copies:
+            t_copy.append(ev[0].elapsed_time(ev[1]) * 1e-3 / len(copies))
+        for pt, _, _ in plans:
+            pool.free(pt)
+    st = nexus.device_status(stream)
+    if st != nexus.OK:
+        raise RuntimeError(f"device status after the arena timing: {nexus.status_string(st)}")
+    p50 = lambda xs: float(np.median(xs)) * 1e6
+    page_bytes = 2.0 * 2 * L * HKV * PAGE * D * 2     # K and V of one page, read + written
+    copy_us = p50(t_copy)
+    out = {"slots": n_slots, "layers": L,
+           "setup": f"{n_slots} slots: a shared {system_len}-token prompt + a {tail_len}-token "
+                    f"tail each; requests fork {system_len} + U[1, {tail_len}) warm tokens",
+           "match_us_p50": p50(t_match), "fork_host_us_p50": p50(t_fork),
+           "copy_us_mean": copy_us, "fork_e2e_us_p50": p50(t_e2e),
+           "timing": "match / fork / e2e: wall clock through the Python binding, one request "
+                     "at a time (e2e ends when the copy has run); copy: CUDA events over 40 "
+                     "back-to-back boundary copies",
+           "roofline": {"bound": "hbm", "kernel": "page_copy_kernel (one boundary page, "
+                                                 f"{L} layers, K and V)",
+                        "achieved": page_bytes / (copy_us * 1e-6) / 1e9, "peak": peaks["hbm_gbs"],
+                        "unit": "GB/s", "frac": page_bytes / (copy_us * 1e-6) / 1e9 / peaks["hbm_gbs"],
+                        "peak_kind": f"copy, {peak_kind}", "traffic": None,
+                        "note": "6.3 MB per launch: too small to reach the HBM bound"}}
+    arena.close(pool)
+    del kp, vp
+    # warm-hit rate on a seeded agent stream (host only)
+    pool2 = nexus.PagePool(1 << 16)
+    ar2 = nexus.WarmArena(n_slots, 1 << 14)
+    hits = reused = total = 0
+    for q in agent_requests(11, 2000, n_agents=48, sys_len=600, vocab=32000):
+        slot, m = ar2.match(q)
+        npg = -(-len(q) // PAGE)
+        pre = np.zeros(0, np.int32)
+        if slot >= 0:
+            pre, _, _ = ar2.fork(pool2, slot, m, npg)
+            hits += m > 0
+        pt = np.concatenate([pre, pool2.alloc(npg - len(pre))]).astype(np.int32)
+        ar2.store(pool2, q, pt)
+        pool2.free(pt)
+        reused += m
+        total += len(q)
+    ar2.close(pool2)
+    out["hit_rate"] = hits / 2000.0
+    out["token_reuse"] = reused / total
+    out["hit_stream"] = "2000 seeded requests of 48 agents sharing a 600-token prompt"
+    if with_oracle:
+        import oracle
+        model = oracle.WarmArenaModel(n_slots, system_len + tail_len)
+        for s in range(n_slots):
+            z = np.zeros((1, system_len + tail_len, 1, 1))
+            model.store(system + tails[s], z, z)
+        q = system + tails[0][:500] + [32001]
+        t0 = time.perf_counter()
+        reps = 3
+        for _ in range(reps):
+            model.match(q)
+        dt = (time.perf_counter() - t0) / reps
+        out["cpu_baseline"] = {"value": dt * 1e6, "unit": "us per match", "cores": 1,
+                               "kind": "oracle",
+                               "sample": f"plain-Python model: one {len(q)}-token query against "
+                                         f"the same {n_slots} slots"}
     return out
 
 

@@ -357,29 +357,71 @@ __global__ void __launch_bounds__(kThreads) splice_kernel(const __grid_constant_
   }
 }
 
-__global__ void __launch_bounds__(kThreads) page_copy_kernel(const __grid_constant__ PageCopyLaunch p) {
-  const int pair = blockIdx.x % p.n;
-  const int layer = p.layer_begin + blockIdx.x / p.n;
-  const int64_t page_vec = (int64_t)p.n_kv_heads * kPageSize * kHeadDim / 8;   // uint4 per page
-  const int64_t so = ((int64_t)layer * p.n_pages + p.src[pair]) * page_vec;
-  const int64_t d_o = ((int64_t)layer * p.n_pages + p.dst[pair]) * page_vec;
+// Whole-page copies (K and V, every layer of the call). One CTA moves two heads
+// of one page pair in one layer (16 KiB of K and V in, 16 KiB out), so even a
+// single pair spreads over layers x heads / 2 CTAs. The pair list travels in the
+// kernel arguments; a short list uses a small argument block, which launches faster.
+template <int kCap>
+struct PageCopyArgs {
+  uint16_t* k_pool;
+  uint16_t* v_pool;
+  int64_t n_pages;
+  int32_t n_kv_heads;
+  int32_t layer_begin;
+  int32_t n_layers_call;
+  int32_t n;
+  int32_t src[kCap];
+  int32_t dst[kCap];
+};
+
+template <int kCap>
+__global__ void __launch_bounds__(kThreads) page_copy_kernel(const __grid_constant__ PageCopyArgs<kCap> p) {
+  constexpr int kHeadVec = kPageSize * kHeadDim / 8;   // uint4 per head of a page
+  const int head_pairs = (p.n_kv_heads + 1) / 2;
+  int b = blockIdx.x;
+  const int hp = b % head_pairs;
+  b /= head_pairs;
+  const int pair = b % p.n;
+  const int layer = p.layer_begin + b / p.n;
+  const int64_t page_vec = (int64_t)p.n_kv_heads * kHeadVec;
+  const int64_t so = ((int64_t)layer * p.n_pages + p.src[pair]) * page_vec + hp * 2 * kHeadVec;
+  const int64_t d_o = ((int64_t)layer * p.n_pages + p.dst[pair]) * page_vec + hp * 2 * kHeadVec;
+  const int nvec = min(2, p.n_kv_heads - 2 * hp) * kHeadVec;
   const uint4* sk = reinterpret_cast<const uint4*>(p.k_pool) + so;
   const uint4* sv = reinterpret_cast<const uint4*>(p.v_pool) + so;
   uint4* dk = reinterpret_cast<uint4*>(p.k_pool) + d_o;
   uint4* dv = reinterpret_cast<uint4*>(p.v_pool) + d_o;
-  for (int64_t i = threadIdx.x; i < page_vec; i += 4 * kThreads) {
-    uint4 a[4], b[4];
+  uint4 a[2], c[2];
 #pragma unroll
-    for (int u = 0; u < 4; ++u) {
-      const int64_t j = i + u * kThreads;
-      if (j < page_vec) { a[u] = sk[j]; b[u] = sv[j]; }
-    }
-#pragma unroll
-    for (int u = 0; u < 4; ++u) {
-      const int64_t j = i + u * kThreads;
-      if (j < page_vec) { dk[j] = a[u]; dv[j] = b[u]; }
-    }
+  for (int u = 0; u < 2; ++u) {
+    const int j = threadIdx.x + u * kThreads;
+    if (j < nvec) { a[u] = sk[j]; c[u] = sv[j]; }
   }
+#pragma unroll
+  for (int u = 0; u < 2; ++u) {
+    const int j = threadIdx.x + u * kThreads;
+    if (j < nvec) { dk[j] = a[u]; dv[j] = c[u]; }
+  }
+}
+
+template <int kCap>
+cudaError_t launch_page_copy_as(const PageCopyLaunch& p, cudaStream_t stream) {
+  PageCopyArgs<kCap> a;
+  a.k_pool = p.k_pool;
+  a.v_pool = p.v_pool;
+  a.n_pages = p.n_pages;
+  a.n_kv_heads = p.n_kv_heads;
+  a.layer_begin = p.layer_begin;
+  a.n_layers_call = p.n_layers_call;
+  a.n = p.n;
+  for (int i = 0; i < p.n; ++i) {
+    a.src[i] = p.src[i];
+    a.dst[i] = p.dst[i];
+  }
+  const int64_t blocks = (int64_t)p.n * p.n_layers_call * ((p.n_kv_heads + 1) / 2);
+  if (blocks > 0x7FFFFFFFLL) return cudaErrorInvalidValue;
+  page_copy_kernel<kCap><<<(unsigned)blocks, kThreads, 0, stream>>>(a);
+  return cudaGetLastError();
 }
 
 }  // namespace
@@ -400,8 +442,8 @@ cudaError_t launch_splice(const SpliceLaunch& p, cudaStream_t stream) {
 
 cudaError_t launch_page_copy(const PageCopyLaunch& p, cudaStream_t stream) {
   if (p.n <= 0 || p.n_layers_call <= 0) return cudaSuccess;
-  page_copy_kernel<<<(unsigned)(p.n * p.n_layers_call), kThreads, 0, stream>>>(p);
-  return cudaGetLastError();
+  if (p.n <= 8) return launch_page_copy_as<8>(p, stream);
+  return launch_page_copy_as<kMaxPageCopies>(p, stream);
 }
 
 }  // namespace nexus

@@ -165,3 +165,27 @@ def qkv_weights(n_heads: int, hidden: int, seed: int, device="cpu", bias: bool =
         g.manual_seed(int(seed) * 1_000_003 + 7)
         b = torch.randn((n_heads * HEAD_DIM,), generator=g, device=device, dtype=torch.float32) * 0.5
     return w, b
+
+
+def agent_requests(seed: int, n_requests: int, n_agents: int = 6, sys_len: int = 300,
+                   vocab: int = 50):
+    """Token sequences of agent requests, seeded: agents share one system prompt;
+    each request extends one agent's history by a reply and a new message; now
+    and then an agent starts a new conversation or its history diverges inside
+    its last turn (an edit). Yields lists of int token ids."""
+    r = _rng(seed)
+    system = [int(t) for t in r.integers(0, vocab, sys_len)]
+
+    def fresh():
+        return system + [int(t) for t in r.integers(0, vocab, int(r.integers(5, 40)))]
+
+    hist = [fresh() for _ in range(n_agents)]
+    for _ in range(n_requests):
+        a = int(r.integers(0, n_agents))
+        if r.random() < 0.1:
+            hist[a] = fresh()
+        elif r.random() < 0.15:
+            cut = max(len(system), len(hist[a]) - int(r.integers(1, 30)))
+            hist[a] = hist[a][:cut] + [int(t) for t in r.integers(vocab, vocab + 10, 4)]
+        hist[a] = hist[a] + [int(t) for t in r.integers(0, vocab, int(r.integers(1, 60)))]
+        yield list(hist[a])

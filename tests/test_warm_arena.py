@@ -13,6 +13,7 @@ import pytest
 
 import oracle
 from paper_2608_20397_gb300 import nexus
+from paper_2608_20397_gb300.workloads import agent_requests
 
 PAGE = 16
 
@@ -53,22 +54,8 @@ class PageStore:
         return np.asarray([self.rows[pt[p // PAGE], p % PAGE] for p in range(n)])
 
 
-def agent_stream(seed, n_requests, n_agents=6, sys_len=300):
-    """Requests of agents sharing a system prompt; each turn extends the
-    agent's history with a reply and a new message; some requests start fresh."""
-    r = np.random.default_rng(seed)
-    system = [int(t) for t in r.integers(0, 50, sys_len)]
-    hist = [list(system) + [int(t) for t in r.integers(0, 50, int(r.integers(5, 40)))]
-            for _ in range(n_agents)]
-    for _ in range(n_requests):
-        a = int(r.integers(0, n_agents))
-        if r.random() < 0.1:   # a new conversation of this agent
-            hist[a] = list(system) + [int(t) for t in r.integers(0, 50, int(r.integers(5, 40)))]
-        elif r.random() < 0.15:   # an edit: the history diverges inside the last turn
-            cut = max(len(system), len(hist[a]) - int(r.integers(1, 30)))
-            hist[a] = hist[a][:cut] + [int(t) for t in r.integers(50, 60, 4)]
-        hist[a] = hist[a] + [int(t) for t in r.integers(0, 50, int(r.integers(1, 60)))]
-        yield list(hist[a])
+def agent_stream(seed, n_requests):
+    return agent_requests(seed, n_requests)
 
 
 def run_stream(n_slots, max_tokens, seed, n_requests, n_pages=4096):
