@@ -489,3 +489,92 @@ def pin_warm_arena(WarmArenaModel):
     arena.store(F, *rows(F))
     arena.store([6000], *rows([6000]))
     assert np.array_equal(k_before, rows(E)[0][:, :120])
+
+
+def pin_slb_quantize(slb_quantize):
+    """INT8 codes of the tool scan (Sec. IV-A): within [-127, 127], the largest
+    magnitude at +-127, reconstruction within half a step, vectors already on the
+    grid unchanged, halves rounded to even, a zero vector left at zero."""
+    r = _rs(25)
+    x = r.standard_normal((20, 96)).astype(np.float32)
+    codes, scales = slb_quantize(x)
+    assert codes.dtype == np.int8 and scales.dtype == np.float32
+    assert np.all(np.abs(codes.astype(int)) <= 127)
+    for i in range(20):
+        j = int(np.argmax(np.abs(x[i])))
+        assert abs(int(codes[i, j])) == 127 and np.sign(codes[i, j]) == np.sign(x[i, j])
+        err = np.abs(x[i].astype(np.float64) - codes[i].astype(np.float64) * float(scales[i]))
+        assert np.all(err <= 0.5 * float(scales[i]) * (1 + 1e-5))
+    g = (r.integers(-127, 128, (5, 64)).astype(np.float32)) * np.float32(0.25)
+    g[:, 0] = np.float32(127 * 0.25)
+    c2, s2 = slb_quantize(g)
+    assert np.all(s2 == np.float32(0.25)) and np.array_equal(c2.astype(np.float32) * 0.25, g)
+    h = np.zeros((1, 4), np.float32)
+    h[0] = [127.0, 2.5, 3.5, -2.5]                    # scale exactly 1
+    c3, _ = slb_quantize(h)
+    assert list(c3[0]) == [127, 2, 4, -2]
+    c4, s4 = slb_quantize(np.zeros((1, 8), np.float32))
+    assert s4[0] == 0 and not c4.any()
+
+
+def pin_slb_scores(slb_scores, slb_quantize):
+    """Scores: a one-hot query code reads one code of each tool times both scales;
+    swapping query and tool changes nothing; for unit vectors the score is the
+    cosine up to the quantization error, sqrt(d) (s_q + s_t) / 2 + s_q s_t d / 4."""
+    r = _rs(26)
+    tc = r.integers(-127, 128, (7, 32)).astype(np.int8)
+    ts = (r.random(7).astype(np.float32) + np.float32(0.5)) * np.float32(0.01)
+    for k in (0, 5, 31):
+        qc = np.zeros((1, 32), np.int8)
+        qc[0, k] = 1
+        got = slb_scores(qc, np.array([1.0], np.float32), tc, ts)[0]
+        want = np.array([np.float32(np.float32(tc[j, k]) * ts[j]) for j in range(7)])
+        assert np.array_equal(got, want)
+    a = slb_scores(tc[:3], ts[:3], tc[3:], ts[3:])
+    b = slb_scores(tc[3:], ts[3:], tc[:3], ts[:3])
+    assert np.array_equal(a, b.T)
+    d = 768
+    x = r.standard_normal((12, d))
+    x /= np.linalg.norm(x, axis=1, keepdims=True)
+    y = x[:4] + 0.3 * r.standard_normal((4, d))
+    y /= np.linalg.norm(y, axis=1, keepdims=True)
+    xc, xs = slb_quantize(x)
+    yc, ys = slb_quantize(y)
+    s = slb_scores(yc, ys, xc, xs)
+    cos = y @ x.T
+    for a_ in range(4):
+        for b_ in range(12):
+            bound = (np.sqrt(d) * (ys[a_] + xs[b_]) / 2 + ys[a_] * xs[b_] * d / 4) * (1 + 1e-6)
+            assert abs(float(s[a_, b_]) - cos[a_, b_]) <= bound
+
+
+def pin_slb_route(slb_route):
+    """The gate: the best two by score then index (brute force over a hand-made
+    registry with a tie), routing only when the margin is strictly above tau,
+    and a lone tool always routed."""
+    one = np.array([1.0], np.float32)
+    q = np.zeros((1, 4), np.int8)
+    q[0, 0] = 1
+    step = np.float32(1.0 / 1024)
+    def registry(vals):
+        t = np.zeros((len(vals), 4), np.int8)
+        t[:, 0] = vals
+        return t, np.full(len(vals), step, np.float32)
+    tau = np.float32(3.0 / 1024)
+    t, ts = registry([7, 10, 3, 10])               # tie at 10: index 1 before 3
+    (i1, i2, s1, s2, route), = slb_route(q, one, t, ts, tau)
+    assert (i1, i2) == (1, 3) and s1 == s2 == np.float32(10 / 1024) and route == -1
+    t, ts = registry([7, 10, 3])                   # margin 3/1024 == tau: escalates
+    assert slb_route(q, one, t, ts, tau)[0][4] == -1
+    t, ts = registry([6, 10, 3])                   # margin 4/1024 > tau: routes to 1
+    assert slb_route(q, one, t, ts, tau)[0][4] == 1
+    t, ts = registry([-5])                         # a single tool: always routed
+    (i1, i2, s1, s2, route), = slb_route(q, one, t, ts, tau)
+    assert (i1, i2, route) == (0, -1, 0) and s2 == -np.inf
+    r = _rs(27)
+    for _ in range(20):
+        vals = r.integers(-127, 128, 9)
+        t, ts = registry(vals)
+        (i1, i2, _, _, _), = slb_route(q, one, t, ts, tau)
+        order = sorted(range(9), key=lambda j: (-int(vals[j]), j))
+        assert (i1, i2) == (order[0], order[1])

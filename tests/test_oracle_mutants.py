@@ -267,3 +267,46 @@ def test_arena_mutants_caught():
 
     for mut in (EvictsMostRecent, NoExtension):
         assert _fails(P.pin_warm_arena, mut), mut.__name__
+
+
+def test_slb_mutants_caught():
+    def round_half_up(x):
+        codes, scales = oracle.slb_quantize(x)
+        x = np.asarray(x, np.float32)
+        for i in range(x.shape[0]):
+            if scales[i]:
+                codes[i] = np.clip(np.floor(x[i] / scales[i] + np.float32(0.5)), -127, 127)
+        return codes, scales
+
+    def scale_by_255(x):
+        x = np.asarray(x, np.float32)
+        codes, scales = oracle.slb_quantize(x)
+        return codes, scales * np.float32(127.0 / 255.0)
+
+    assert _fails(P.pin_slb_quantize, round_half_up)
+    assert _fails(P.pin_slb_quantize, scale_by_255)
+
+    def no_tool_scale(qc, qs, tc, ts):
+        return oracle.slb_scores(qc, qs, tc, np.ones_like(ts))
+
+    assert _fails(P.pin_slb_scores, no_tool_scale, oracle.slb_quantize)
+
+    def gate_inclusive(qc, qs, tc, ts, tau=oracle.slb.TAU):
+        out = []
+        for i1, i2, s1, s2, _ in oracle.slb_route(qc, qs, tc, ts, tau):
+            out.append((i1, i2, s1, s2, i1 if np.float32(s1 - s2) >= tau else -1))
+        return out
+
+    def ties_to_last(qc, qs, tc, ts, tau=oracle.slb.TAU):
+        s = oracle.slb_scores(qc, qs, tc, ts)
+        out = []
+        for a in range(s.shape[0]):
+            order = sorted(range(s.shape[1]), key=lambda j: (-float(s[a, j]), -j))
+            i1 = order[0]
+            i2 = order[1] if len(order) > 1 else -1
+            s2 = s[a, i2] if i2 >= 0 else np.float32(-np.inf)
+            out.append((i1, i2, s[a, i1], s2, i1 if s[a, i1] - s2 > tau else -1))
+        return out
+
+    assert _fails(P.pin_slb_route, gate_inclusive)
+    assert _fails(P.pin_slb_route, ties_to_last)

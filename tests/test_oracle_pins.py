@@ -91,3 +91,15 @@ def test_warm_match():
 
 def test_warm_arena():
     P.pin_warm_arena(oracle.WarmArenaModel)
+
+
+def test_slb_quantize():
+    P.pin_slb_quantize(oracle.slb_quantize)
+
+
+def test_slb_scores():
+    P.pin_slb_scores(oracle.slb_scores, oracle.slb_quantize)
+
+
+def test_slb_route():
+    P.pin_slb_route(oracle.slb_route)
