@@ -55,13 +55,10 @@ def slb_scores(q_codes, q_scales, t_codes, t_scales) -> np.ndarray:
     """float32 scores [n_queries][n_tools] of the rule above."""
     qc = np.asarray(q_codes, dtype=np.int64)
     tc = np.asarray(t_codes, dtype=np.int64)
-    out = np.zeros((qc.shape[0], tc.shape[0]), dtype=np.float32)
-    for a in range(qc.shape[0]):
-        for b in range(tc.shape[0]):
-            dot = int(np.sum(qc[a] * tc[b]))
-            c = np.float32(np.float32(q_scales[a]) * np.float32(t_scales[b]))
-            out[a, b] = np.float32(np.float32(dot) * c)
-    return out
+    dots = qc @ tc.T                                   # exact integer dot products
+    c = (np.asarray(q_scales, dtype=np.float32)[:, None] *
+         np.asarray(t_scales, dtype=np.float32)[None, :])   # float32 products of the scales
+    return dots.astype(np.float32) * c
 
 
 def slb_top2(scores_row) -> List[Tuple[int, np.float32]]:
