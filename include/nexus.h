@@ -29,6 +29,8 @@
  *                            copy-on-write) and splice planner
  *   nexus_warm_arena_*       the L0 exact-token radix arena of warm prefixes
  *                            (Sec. V-D)
+ *   nexus_slb_*              INT8 tool scan with the top-2 margin gate of the
+ *                            semantic lookaside buffer (Sec. IV-A)
  *
  * Conventions
  *   - Device buffers are owned by the caller. The library never allocates or
@@ -422,6 +424,38 @@ nexus_status nexus_suffix_qkv(const nexus_kv_cache* cache, const int32_t* d_page
                               const int32_t* h_q_len, const void* x, int32_t hidden,
                               const void* w_qkv, const float* b_qkv, int32_t n_q_heads,
                               int32_t layer, void* q_out, nexus_stream stream);
+
+/* ------------------------------------------------- INT8 tool scan + gate */
+/* INT8 quantisation of embeddings for the tool scan (Sec. IV-A), on the host:
+ * per row of h_x [n][dim] (finite floats), scale = max|x| / 127 and code =
+ * round-half-even(x / scale) in [-127, 127], in float32; an all-zero row gets
+ * scale 0 and zero codes. NEXUS_EINVAL for a non-finite input. */
+nexus_status nexus_slb_quantize(const float* h_x, int32_t n, int32_t dim, int8_t* h_codes,
+                                float* h_scales);
+/* Bytes of workspace nexus_slb_route needs for a registry of n_tools. */
+size_t nexus_slb_workspace_size(int32_t n_tools);
+/* The semantic lookaside buffer's scan and margin gate (Sec. IV-A): for every
+ * query q, score(q, t) = float(dot(codes_q, codes_t)) * (scale_q * scale_t)
+ * over all tools t (float32; the integer dot is exact), the two best tools
+ * (higher score first, then lower index) and their scores, and the decision:
+ * route[q] = the best tool when top1 - top2 > tau, else -1 (escalate to the
+ * cross-encoder, which is not part of this library). With one tool the
+ * runner-up is index -1 with score -inf and the query always routes.
+ *   d_tools     device int8 [n_tools][dim], dim a multiple of 4 (<= 4096),
+ *               16-byte aligned; d_tool_scales float [n_tools]
+ *   d_queries   device int8 [n_queries][dim], d_query_scales float [n_queries]
+ *   d_top_idx   device int32 [n_queries][2]; d_top_score float [n_queries][2];
+ *               d_route int32 [n_queries]
+ *   workspace   device, nexus_slb_workspace_size(n_tools) bytes, 16-byte
+ *               aligned, all zero before its first use; every call leaves it
+ *               ready for the next (calls sharing one workspace must be ordered
+ *               on the GPU, e.g. by one stream)
+ * Queries are scanned 32 per launch. tau (e.g. 0.0136) must be finite. */
+nexus_status nexus_slb_route(const int8_t* d_tools, const float* d_tool_scales, int32_t n_tools,
+                             int32_t dim, const int8_t* d_queries, const float* d_query_scales,
+                             int32_t n_queries, float tau, int32_t* d_top_idx, float* d_top_score,
+                             int32_t* d_route, void* workspace, size_t workspace_bytes,
+                             nexus_stream stream);
 
 /* Bytes of workspace nexus_suffix_attention needs for these arguments
  * (0 when no split is used). *splits_out (nullable) receives the partition

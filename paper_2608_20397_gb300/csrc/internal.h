@@ -155,4 +155,25 @@ cudaError_t launch_qkv(const QkvLaunch& p, const QkvMaps& maps, int grid, cudaSt
 // a page id outside the pool.
 cudaError_t qkv_take_status(unsigned int* timeout, unsigned int* bad_page, cudaStream_t stream);
 
+// ----------------------------------------------------- INT8 tool scan + gate
+struct SlbLaunch {
+  const int8_t* tools;          // [n_tools][dim]
+  const float* tool_scales;     // [n_tools]
+  const int8_t* queries;        // [n_queries][dim] (this launch's queries)
+  const float* query_scales;    // [n_queries]
+  int32_t* top_idx;             // [n_queries][2]
+  float* top_score;             // [n_queries][2]
+  int32_t* route;               // [n_queries]
+  float* part_score;            // workspace [grid][32][2]
+  int32_t* part_idx;            // workspace [grid][32][2]
+  unsigned int* counter;        // workspace ticket, 0 between calls
+  int32_t n_tools;
+  int32_t dim;                  // multiple of 4
+  int32_t n_queries;            // 1..32
+  int32_t tools_per_cta;
+  float tau;
+};
+constexpr int kSlbMaxQueries = 32;
+cudaError_t launch_slb(const SlbLaunch& p, int grid, cudaStream_t stream);
+
 }  // namespace nexus

@@ -250,6 +250,16 @@ bool encode_2d_sw128(CUtensorMap* m, const void* base, uint64_t inner, uint64_t 
   return r == CUDA_SUCCESS;
 }
 
+// Tool scan: CTAs of 8 warps, about 64 tools per CTA, at most two waves.
+constexpr size_t kSlbPartOffset = 256;
+int slb_grid(int32_t n_tools, int32_t* per_out) {
+  int grid = static_cast<int>(std::min<int64_t>((n_tools + 63) / 64, 2 * num_sms()));
+  grid = std::max(grid, 1);
+  const int32_t per = (n_tools + grid - 1) / grid;
+  if (per_out) *per_out = per;
+  return (n_tools + per - 1) / per;
+}
+
 struct AttnPlan {
   int32_t total_tiles = 0;
   int32_t n_tok = 0;
@@ -640,6 +650,83 @@ nexus_status nexus_suffix_qkv(const nexus_kv_cache* cache, const int32_t* d_page
   const int grid = static_cast<int>(std::min<int64_t>(total, num_sms()));
   return launch_qkv(*p, maps, grid, static_cast<cudaStream_t>(stream)) == cudaSuccess ? NEXUS_OK
                                                                                       : NEXUS_ECUDA;
+}
+
+size_t nexus_slb_workspace_size(int32_t n_tools) {
+  if (n_tools < 1) return 0;
+  const int grid = slb_grid(n_tools, nullptr);
+  return kSlbPartOffset + static_cast<size_t>(grid) * kSlbMaxQueries * 2 * (sizeof(float) + sizeof(int32_t));
+}
+
+nexus_status nexus_slb_route(const int8_t* d_tools, const float* d_tool_scales, int32_t n_tools,
+                             int32_t dim, const int8_t* d_queries, const float* d_query_scales,
+                             int32_t n_queries, float tau, int32_t* d_top_idx, float* d_top_score,
+                             int32_t* d_route, void* workspace, size_t workspace_bytes,
+                             nexus_stream stream) {
+  if (!d_tools || !d_tool_scales || n_tools < 1 || n_queries < 0 || !std::isfinite(tau))
+    return NEXUS_EINVAL;
+  if (n_queries > 0 && (!d_queries || !d_query_scales || !d_top_idx || !d_top_score || !d_route))
+    return NEXUS_EINVAL;
+  if (dim < 4 || dim > 4096) return NEXUS_EINVAL;
+  if (dim % 4 != 0 || !aligned16(d_tools) || (d_queries && !aligned16(d_queries)))
+    return NEXUS_ELAYOUT;
+  if (reinterpret_cast<uintptr_t>(d_tool_scales) % 4 || reinterpret_cast<uintptr_t>(d_top_idx) % 4 ||
+      reinterpret_cast<uintptr_t>(d_top_score) % 4 || reinterpret_cast<uintptr_t>(d_route) % 4 ||
+      reinterpret_cast<uintptr_t>(d_query_scales) % 4)
+    return NEXUS_ELAYOUT;
+  if (n_queries == 0) return NEXUS_OK;
+  if (!workspace || !aligned16(workspace) || workspace_bytes < nexus_slb_workspace_size(n_tools))
+    return NEXUS_ENOMEM;
+  int32_t per = 0;
+  const int grid = slb_grid(n_tools, &per);
+  uint8_t* ws = static_cast<uint8_t*>(workspace);
+  SlbLaunch p;
+  p.tools = d_tools;
+  p.tool_scales = d_tool_scales;
+  p.n_tools = n_tools;
+  p.dim = dim;
+  p.tools_per_cta = per;
+  p.tau = tau;
+  p.counter = reinterpret_cast<unsigned int*>(ws);
+  p.part_score = reinterpret_cast<float*>(ws + kSlbPartOffset);
+  p.part_idx = reinterpret_cast<int32_t*>(ws + kSlbPartOffset +
+                                          static_cast<size_t>(grid) * kSlbMaxQueries * 2 * sizeof(float));
+  for (int32_t q0 = 0; q0 < n_queries; q0 += kSlbMaxQueries) {
+    p.n_queries = std::min(kSlbMaxQueries, n_queries - q0);
+    p.queries = d_queries + static_cast<int64_t>(q0) * dim;
+    p.query_scales = d_query_scales + q0;
+    p.top_idx = d_top_idx + 2 * static_cast<int64_t>(q0);
+    p.top_score = d_top_score + 2 * static_cast<int64_t>(q0);
+    p.route = d_route + q0;
+    if (launch_slb(p, grid, static_cast<cudaStream_t>(stream)) != cudaSuccess) return NEXUS_ECUDA;
+  }
+  return NEXUS_OK;
+}
+
+nexus_status nexus_slb_quantize(const float* h_x, int32_t n, int32_t dim, int8_t* h_codes,
+                                float* h_scales) {
+  if (n < 0 || dim < 1 || (n > 0 && (!h_x || !h_codes || !h_scales))) return NEXUS_EINVAL;
+  for (int32_t i = 0; i < n; ++i) {
+    const float* x = h_x + static_cast<int64_t>(i) * dim;
+    int8_t* c = h_codes + static_cast<int64_t>(i) * dim;
+    float amax = 0.f;
+    for (int32_t j = 0; j < dim; ++j) {
+      if (!std::isfinite(x[j])) return NEXUS_EINVAL;
+      amax = std::max(amax, std::fabs(x[j]));
+    }
+    if (amax == 0.f) {
+      std::memset(c, 0, static_cast<size_t>(dim));
+      h_scales[i] = 0.f;
+      continue;
+    }
+    const float scale = amax / 127.0f;
+    for (int32_t j = 0; j < dim; ++j) {
+      const float q = std::nearbyint(x[j] / scale);   // ties to even in the default rounding mode
+      c[j] = static_cast<int8_t>(std::min(127.f, std::max(-127.f, q)));
+    }
+    h_scales[i] = scale;
+  }
+  return NEXUS_OK;
 }
 
 size_t nexus_attention_workspace_size(int32_t n_seqs, const int32_t* h_kv_len,

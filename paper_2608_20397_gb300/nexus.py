@@ -95,6 +95,11 @@ _SIGS = {
                                         _i32p, _i32p, _i32p]),
     "nexus_warm_arena_store": (c_int32, [c_void_p, c_void_p, _i32p, c_int32, _i32p, _i32p]),
     "nexus_warm_arena_slot": (c_int32, [c_void_p, c_int32, _i32p, _i32p, c_int32]),
+    "nexus_slb_quantize": (c_int32, [c_void_p, c_int32, c_int32, c_void_p, c_void_p]),
+    "nexus_slb_workspace_size": (c_size_t, [c_int32]),
+    "nexus_slb_route": (c_int32, [c_void_p, c_void_p, c_int32, c_int32, c_void_p, c_void_p,
+                                  c_int32, ctypes.c_float, c_void_p, c_void_p, c_void_p,
+                                  c_void_p, c_size_t, c_void_p]),
     "nexus_plan_splice": (c_int32, [c_void_p, _i32p, c_int32, c_int32, POINTER(Block), c_int32,
                                     POINTER(Insert), c_int32, c_int32, c_int32, _i32p,
                                     POINTER(Segment), c_int32, _i32p, _i32p, _i32p]),
@@ -508,3 +513,30 @@ class WarmArena:
             self.close()
         except Exception:
             pass
+
+
+# ------------------------------------------------------ INT8 tool scan + gate
+def slb_quantize(x: np.ndarray):
+    """Host INT8 quantisation of embedding rows: (codes int8, scales float32)."""
+    x = np.ascontiguousarray(np.asarray(x, dtype=np.float32))
+    n, dim = x.shape
+    codes = np.zeros((n, dim), np.int8)
+    scales = np.zeros(n, np.float32)
+    _check("nexus_slb_quantize", lib().nexus_slb_quantize(
+        x.ctypes.data, int(n), int(dim), codes.ctypes.data, scales.ctypes.data))
+    return codes, scales
+
+
+def slb_workspace_size(n_tools: int) -> int:
+    return int(lib().nexus_slb_workspace_size(int(n_tools)))
+
+
+def slb_route(tools, tool_scales, queries, query_scales, top_idx, top_score, route, workspace,
+              tau: float = 0.0136, stream=None):
+    """Scan and gate on device tensors (see nexus.h): tools int8 [N][dim],
+    queries int8 [Q][dim]; writes top_idx int32 [Q][2], top_score float [Q][2],
+    route int32 [Q]. The workspace (nexus_slb_workspace_size bytes) starts zeroed."""
+    _check("nexus_slb_route", lib().nexus_slb_route(
+        _ptr(tools), _ptr(tool_scales), int(tools.shape[0]), int(tools.shape[1]), _ptr(queries),
+        _ptr(query_scales), int(queries.shape[0]), float(tau), _ptr(top_idx), _ptr(top_score),
+        _ptr(route), _ptr(workspace), int(workspace.numel()), _stream(stream)))

@@ -189,3 +189,30 @@ def agent_requests(seed: int, n_requests: int, n_agents: int = 6, sys_len: int =
             hist[a] = hist[a][:cut] + [int(t) for t in r.integers(vocab, vocab + 10, 4)]
         hist[a] = hist[a] + [int(t) for t in r.integers(0, vocab, int(r.integers(1, 60)))]
         yield list(hist[a])
+
+
+def tool_registry(n_tools: int, dim: int = 768, seed: int = 0, family: int = 5,
+                  spread: float = 0.2):
+    """Unit-norm float32 tool embeddings [n_tools][dim] in families of `family`
+    tools scattered around a shared direction (tools of one server that share
+    words), so that neighbours are close and some top-2 margins are small. With
+    the default spread and query noise, the gate threshold 0.0136 falls near the
+    20th percentile of the top-2 margins of 250 tools, where the paper puts it."""
+    r = _rng(seed)
+    n_fam = -(-n_tools // family)
+    centers = r.standard_normal((n_fam, dim))
+    centers /= np.linalg.norm(centers, axis=1, keepdims=True)
+    x = centers[np.arange(n_tools) // family] + spread * r.standard_normal((n_tools, dim)) / np.sqrt(dim)
+    x /= np.linalg.norm(x, axis=1, keepdims=True)
+    return x.astype(np.float32)
+
+
+def tool_queries(registry: np.ndarray, n_queries: int, seed: int = 1, noise: float = 1.2):
+    """Query embeddings: a tool's embedding plus noise, renormalised; returns
+    (queries float32 [n][dim], the tool each was drawn from)."""
+    r = _rng(seed)
+    n_tools, dim = registry.shape
+    src = r.integers(0, n_tools, n_queries)
+    q = registry[src].astype(np.float64) + noise * r.standard_normal((n_queries, dim)) / np.sqrt(dim)
+    q /= np.linalg.norm(q, axis=1, keepdims=True)
+    return q.astype(np.float32), src

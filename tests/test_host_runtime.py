@@ -346,3 +346,40 @@ def test_qkv_argument_checks():
     shared[1, 2] = shared[0, 2]                           # both rows write page 2's slots
     assert code(kv=(40, 40), ql=(8, 8), rows=[0, 1], hpt=shared, n_rows=2) == nexus.EOVERLAP
     call(kv=(40, 40), ql=(0, 0), rows=[0, 1], hpt=pt, n_rows=2)   # nothing to do: no launch
+
+
+def test_slb_quantize_matches_oracle():
+    r = np.random.default_rng(41)
+    x = r.standard_normal((40, 768)).astype(np.float32) * r.uniform(1e-3, 1e3, (40, 1)).astype(np.float32)
+    x[3] = 0.0
+    x[4, :4] = [127.0, 2.5, -3.5, 0.5]        # scale exactly 1: halves go to even
+    x[4, 4:] = 0.0
+    x[5] = r.integers(-127, 128, 768).astype(np.float32) * np.float32(0.125)
+    c, s = nexus.slb_quantize(x)
+    c2, s2 = oracle.slb_quantize(x)
+    assert np.array_equal(c, c2) and np.array_equal(s, s2)
+    assert list(c[4, :4]) == [127, 2, -4, 0]
+    bad = np.zeros((1, 8), np.float32)
+    bad[0, 1] = np.inf
+    with pytest.raises(nexus.NexusError) as e:
+        nexus.slb_quantize(bad)
+    assert e.value.code == nexus.EINVAL
+
+
+def test_slb_route_argument_checks():
+    L = nexus.lib()
+    ws = nexus.slb_workspace_size(250)
+    assert ws >= 256 + 32 * 2 * 8 and nexus.slb_workspace_size(0) == 0
+    def call(n_tools=250, dim=768, nq=1, tau=0.0136, tools=FAKE, queries=FAKE, ws_bytes=ws,
+             wsp=FAKE):
+        return L.nexus_slb_route(tools, FAKE, n_tools, dim, queries, FAKE, nq, tau, FAKE, FAKE,
+                                 FAKE, wsp, ws_bytes, None)
+    assert call(n_tools=0) == nexus.EINVAL
+    assert call(dim=2) == nexus.EINVAL
+    assert call(dim=8192) == nexus.EINVAL
+    assert call(dim=770) == nexus.ELAYOUT
+    assert call(tools=FAKE + 4) == nexus.ELAYOUT
+    assert call(tau=float("nan")) == nexus.EINVAL
+    assert call(ws_bytes=ws - 1) == nexus.ENOMEM
+    assert call(wsp=None) == nexus.ENOMEM
+    assert call(nq=0) == nexus.OK                # nothing to scan: no launch

@@ -1,0 +1,113 @@
+"""Parity of the INT8 tool scan and top-2 margin gate (Sec. IV-A) with the
+oracle: top-2 indices, their float32 scores and the routing decision, all
+exact (the integer dots are exact and both sides form the scores with the same
+float32 operations).
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2608_20397_gb300 import nexus
+from paper_2608_20397_gb300.workloads import tool_queries, tool_registry
+
+pytestmark = pytest.mark.gpu
+TAU = 0.0136
+
+
+@pytest.fixture(scope="module")
+def dev():
+    if not torch.cuda.is_available():
+        pytest.skip("no GPU")
+    return torch.device("cuda:0")
+
+
+def run(dev, tc, ts, qc, qs, tau=TAU, ws=None):
+    nq = qc.shape[0]
+    d = lambda a: torch.as_tensor(np.ascontiguousarray(a), device=dev)
+    top_idx = torch.full((nq, 2), -7, dtype=torch.int32, device=dev)
+    top_score = torch.full((nq, 2), float("nan"), dtype=torch.float32, device=dev)
+    route = torch.full((nq,), -7, dtype=torch.int32, device=dev)
+    if ws is None:
+        ws = torch.zeros(nexus.slb_workspace_size(tc.shape[0]), dtype=torch.uint8, device=dev)
+    nexus.slb_route(d(tc), d(ts), d(qc), d(qs), top_idx, top_score, route, ws, tau)
+    torch.cuda.synchronize()
+    return top_idx.cpu().numpy(), top_score.cpu().numpy(), route.cpu().numpy()
+
+
+def check(got, tc, ts, qc, qs, tau=TAU):
+    top_idx, top_score, route = got
+    want = oracle.slb_route(qc, qs, tc, ts, np.float32(tau))
+    for a, (i1, i2, s1, s2, r) in enumerate(want):
+        assert (top_idx[a, 0], top_idx[a, 1]) == (i1, i2), a
+        assert top_score[a, 0] == s1 and top_score[a, 1] == s2, a
+        assert route[a] == r, a
+
+
+def test_slb_paper_size(dev):
+    # 250 tools x 768 dims; 33 queries: a full launch of 32 and one more
+    x = tool_registry(250)
+    q, _ = tool_queries(x, 33)
+    tc, ts = oracle.slb_quantize(x)
+    qc, qs = oracle.slb_quantize(q)
+    got = run(dev, tc, ts, qc, qs)
+    check(got, tc, ts, qc, qs)
+    assert 0 < np.mean(got[2] == -1) < 1          # some queries escalate, some route
+
+
+@pytest.mark.parametrize("nq", [1, 3, 8, 16, 32])
+def test_slb_query_batches(dev, nq):
+    x = tool_registry(1000, seed=4)
+    q, _ = tool_queries(x, nq, seed=5)
+    tc, ts = oracle.slb_quantize(x)
+    qc, qs = oracle.slb_quantize(q)
+    check(run(dev, tc, ts, qc, qs), tc, ts, qc, qs)
+
+
+def test_slb_edge_cases(dev):
+    r = np.random.default_rng(6)
+    # a single tool: no runner-up, always routed
+    tc = r.integers(-127, 128, (1, 64)).astype(np.int8)
+    ts = np.array([0.01], np.float32)
+    qc = r.integers(-127, 128, (3, 64)).astype(np.int8)
+    qs = np.full(3, 0.02, np.float32)
+    got = run(dev, tc, ts, qc, qs)
+    check(got, tc, ts, qc, qs)
+    assert list(got[0][:, 1]) == [-1] * 3 and list(got[2]) == [0] * 3
+    # identical tools tie: the lower index ranks first and the zero margin escalates
+    tc2 = np.repeat(tc, 5, axis=0)
+    got = run(dev, tc2, np.full(5, 0.01, np.float32), qc, qs)
+    check(got, tc2, np.full(5, 0.01, np.float32), qc, qs)
+    assert list(got[0][:, 0]) == [0] * 3 and list(got[0][:, 1]) == [1] * 3
+    assert list(got[2]) == [-1] * 3
+    # dim 4, and a zero query (every score 0)
+    tc3 = r.integers(-127, 128, (37, 4)).astype(np.int8)
+    ts3 = r.random(37).astype(np.float32)
+    qc3 = np.zeros((2, 4), np.int8)
+    qc3[1] = [1, -2, 3, -4]
+    qs3 = np.array([0.0, 0.5], np.float32)
+    check(run(dev, tc3, ts3, qc3, qs3), tc3, ts3, qc3, qs3)
+
+
+def test_slb_wide_rows(dev):
+    # dim 4096 with 32 queries: 128 KiB of queries in shared memory
+    x = tool_registry(300, dim=4096, seed=8)
+    q, _ = tool_queries(x, 32, seed=9)
+    tc, ts = oracle.slb_quantize(x)
+    qc, qs = oracle.slb_quantize(q)
+    check(run(dev, tc, ts, qc, qs), tc, ts, qc, qs)
+
+
+def test_slb_large_registry_and_workspace_reuse(dev):
+    # 100000 tools (77 MB of codes, several waves of CTAs); two calls on one workspace
+    x = tool_registry(100_000, seed=10)
+    q, _ = tool_queries(x, 40, seed=11)
+    tc, ts = oracle.slb_quantize(x)
+    qc, qs = oracle.slb_quantize(q)
+    ws = torch.zeros(nexus.slb_workspace_size(tc.shape[0]), dtype=torch.uint8, device=dev)
+    first = run(dev, tc, ts, qc, qs, ws=ws)
+    check(first, tc, ts, qc, qs)
+    second = run(dev, tc, ts, qc, qs, ws=ws)
+    for a, b in zip(first, second):
+        assert np.array_equal(a, b)
+    assert not ws[:16].any()                        # the ticket is back at zero
