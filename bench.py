@@ -17,7 +17,8 @@ causal-visible flops 4 d Hq (R (T - R) + R (R + 1) / 2) per layer), with the
 splice GB/s (8192 algorithmic bytes per moved token-layer) beside it. The fresh
 Q/K/V of re-decoded tokens (projection + RoPE + cache write) is timed apart from
 the step under "qkv_recompute" (2 x 5120 x 7168 flops per token), and the L0
-warm arena (prefix match, fork, one boundary-page copy) under "l0_arena".
+warm arena (prefix match, fork, one boundary-page copy) under "l0_arena", and the
+INT8 tool scan with its margin gate under "slb_route".
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
 
@@ -305,9 +306,11 @@ def main():
                     help="skip the separate timing of the suffix Q/K/V recompute")
     ap.add_argument("--no-arena", action="store_true",
                     help="skip the separate timing of the L0 warm arena")
+    ap.add_argument("--no-slb", action="store_true",
+                    help="skip the separate timing of the INT8 tool scan")
     ap.add_argument("--layers", type=int, default=48, help="layers of the workload (48 = c5)")
     ap.add_argument("--profile", choices=["reprefill", "reprefill-softcap", "splice", "suffix",
-                                          "qkv"],
+                                          "qkv", "slb"],
                     default=None,
                     help="run only this kernel of the step (small case for ncu captures)")
     ap.add_argument("--workload", choices=["c5", "c3"], default="c5",
@@ -408,6 +411,11 @@ def main():
         arena = _arena_measure(wl, stream, peaks, peak_kind,
                                with_oracle=rank == 0 and world == 1 and not args.no_cpu_baseline)
 
+    slb = None
+    if not args.no_slb:
+        slb = _slb_measure(wl, stream, peaks, peak_kind,
+                           with_oracle=rank == 0 and world == 1 and not args.no_cpu_baseline)
+
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         f64 = lambda t: t.float().cpu().double().numpy()
@@ -432,7 +440,7 @@ def main():
             "splice_gbs": splice_gbs, "splice_ms": splice_ms, "reprefill_ms": pre_ms,
             "suffix_ms": suf_ms, "suffix_tflops": suf_tflops,
             "roofline": roofline, "roofline_splice": roofline_splice,
-            "e2e": e2e, "cpu_baseline": cpu, "clocks": clocks, "qkv_recompute": qkv, "l0_arena": arena,
+            "e2e": e2e, "cpu_baseline": cpu, "clocks": clocks, "qkv_recompute": qkv, "l0_arena": arena, "slb_route": slb,
             "gpu_launches": wl.launches_per_step * args.steps,
         }
         print(json.dumps(line), flush=True)
@@ -460,8 +468,26 @@ def _profile_only(wl, args, stream):
         qkv_q = torch.empty((qkv_n, HQ, D), dtype=torch.bfloat16, device=dev)
         qkv_flops = 2.0 * qkv_n * HIDDEN * (HQ + 2 * HKV) * D
 
+    if args.profile == "slb":
+        # the 1M-tool registry of the bench's large tool scan, 32 queries per launch
+        dev = wl.kp.device
+        g = torch.Generator(device=dev)
+        g.manual_seed(12)
+        slb_t = torch.randint(-127, 128, (1 << 20, 768), generator=g, device=dev,
+                              dtype=torch.int32).to(torch.int8)
+        slb_ts = torch.rand(1 << 20, generator=g, device=dev) * 0.01
+        slb_q = torch.randint(-127, 128, (32, 768), generator=g, device=dev,
+                              dtype=torch.int32).to(torch.int8)
+        slb_qs = torch.rand(32, generator=g, device=dev) * 0.01
+        slb_ws = torch.zeros(nexus.slb_workspace_size(1 << 20), dtype=torch.uint8, device=dev)
+        slb_out = (torch.empty((32, 2), dtype=torch.int32, device=dev),
+                   torch.empty((32, 2), dtype=torch.float32, device=dev),
+                   torch.empty(32, dtype=torch.int32, device=dev))
+
     def one():
-        if args.profile == "qkv":
+        if args.profile == "slb":
+            nexus.slb_route(slb_t, slb_ts, slb_q, slb_qs, *slb_out, slb_ws, stream=stream)
+        elif args.profile == "qkv":
             nexus.suffix_qkv(wl.cache, wl.d_pt, 2, wl.max_pages, [qkv_kv], [qkv_n], qkv_x, qkv_w,
                              qkv_b, qkv_q, layer=0, n_q_heads=HQ, rows=[qkv_row], stream=stream)
         elif args.profile == "splice":
@@ -494,6 +520,14 @@ def _profile_only(wl, args, stream):
     torch.cuda.synchronize()
     st = nexus.device_status(stream)
     ms = a.elapsed_time(b) / args.steps
+    if args.profile == "slb":
+        gbs = (1 << 20) * 772.0 / (ms * 1e-3) / 1e9
+        print(json.dumps({"profile": "slb", "tools": 1 << 20, "ms_per_launch": ms,
+                          "rate": f"{gbs:.1f} GB/s", "status": nexus.status_string(st)}),
+              flush=True)
+        if st != nexus.OK:
+            raise SystemExit(1)
+        return
     if args.profile == "qkv":
         print(json.dumps({"profile": "qkv", "workload": args.workload, "tokens": qkv_n,
                           "ms_per_launch": ms,
@@ -707,6 +741,110 @@ def _arena_measure(wl, stream, peaks, peak_kind, with_oracle, n_slots=32, system
                                "kind": "oracle",
                                "sample": f"plain-Python model: one {len(q)}-token query against "
                                          f"the same {n_slots} slots"}
+    return out
+
+
+def _slb_measure(wl, stream, peaks, peak_kind, with_oracle, reps=200):
+    """The INT8 tool scan and margin gate (Sec. IV-A), timed apart from the step:
+    (a) the paper's size, 250 tools x 768 dims, one query: the kernel alone
+    (CUDA events over back-to-back launches enqueued behind a fixed sleep) and a
+    whole routing call from a host embedding (quantise, copy in, scan, copy the
+    decision out, P50); (b) a registry of 1M tools (768 MB of codes, larger than
+    L2), 32 queries per launch, against the HBM roofline."""
+    import torch
+
+    from paper_2608_20397_gb300.workloads import tool_queries, tool_registry
+    nexus = wl.nexus
+    dev = wl.kp.device
+    x = tool_registry(250)
+    q, _ = tool_queries(x, reps + 10)
+    tc, ts = nexus.slb_quantize(x)
+    d_tc = torch.as_tensor(tc, device=dev)
+    d_ts = torch.as_tensor(ts, device=dev)
+    ws = torch.zeros(nexus.slb_workspace_size(250), dtype=torch.uint8, device=dev)
+    top_idx = torch.empty((32, 2), dtype=torch.int32, device=dev)
+    top_score = torch.empty((32, 2), dtype=torch.float32, device=dev)
+    route = torch.empty(32, dtype=torch.int32, device=dev)
+    h_qc = torch.empty((1, 768), dtype=torch.int8, pin_memory=True)
+    h_qs = torch.empty(1, dtype=torch.float32, pin_memory=True)
+    h_out = torch.empty(3, dtype=torch.int32, pin_memory=True)
+    d_qc = torch.empty((1, 768), dtype=torch.int8, device=dev)
+    d_qs = torch.empty(1, dtype=torch.float32, device=dev)
+    t_e2e = []
+    for i in range(reps + 10):
+        stream.synchronize()
+        t0 = time.perf_counter()
+        qc, qs = nexus.slb_quantize(q[i:i + 1])
+        h_qc.numpy()[:] = qc
+        h_qs.numpy()[:] = qs
+        d_qc.copy_(h_qc, non_blocking=True)
+        d_qs.copy_(h_qs, non_blocking=True)
+        nexus.slb_route(d_tc, d_ts, d_qc, d_qs, top_idx[:1], top_score[:1], route[:1], ws,
+                        stream=stream)
+        h_out[:2].copy_(top_idx[0], non_blocking=True)
+        h_out[2:].copy_(route[:1], non_blocking=True)
+        stream.synchronize()
+        if i >= 10:
+            t_e2e.append(time.perf_counter() - t0)
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
+    def kernel_us(tools, scales, queries, qscales, n_launch, w):
+        torch.cuda._sleep(4_000_000)
+        ev[0].record(stream)
+        for _ in range(n_launch):
+            nexus.slb_route(tools, scales, queries, qscales, top_idx[:queries.shape[0]],
+                            top_score[:queries.shape[0]], route[:queries.shape[0]], w,
+                            stream=stream)
+        ev[1].record(stream)
+        ev[1].synchronize()
+        return ev[0].elapsed_time(ev[1]) * 1e3 / n_launch
+    kernel_us(d_tc, d_ts, d_qc, d_qs, 10, ws)
+    small_us = float(np.median([kernel_us(d_tc, d_ts, d_qc, d_qs, 50, ws) for _ in range(5)]))
+    # 1M tools: codes and scales drawn on the device (the scan's time does not
+    # depend on the values)
+    n_big, dim = 1 << 20, 768
+    g = torch.Generator(device=dev)
+    g.manual_seed(12)
+    big = torch.randint(-127, 128, (n_big, dim), generator=g, device=dev, dtype=torch.int32).to(torch.int8)
+    big_s = torch.rand(n_big, generator=g, device=dev) * 0.01
+    bq = torch.randint(-127, 128, (32, dim), generator=g, device=dev, dtype=torch.int32).to(torch.int8)
+    bqs = torch.rand(32, generator=g, device=dev) * 0.01
+    ws_big = torch.zeros(nexus.slb_workspace_size(n_big), dtype=torch.uint8, device=dev)
+    big_bytes = n_big * (dim + 4.0)
+    by_batch = {}
+    for nb in (1, 8, 32):
+        kernel_us(big, big_s, bq[:nb], bqs[:nb], 2, ws_big)
+        us = float(np.median([kernel_us(big, big_s, bq[:nb], bqs[:nb], 5, ws_big)
+                              for _ in range(3)]))
+        by_batch[nb] = {"kernel_us": us, "gbs": big_bytes / (us * 1e-6) / 1e9,
+                        "queries_per_s": nb / (us * 1e-6)}
+    big_us = by_batch[32]["kernel_us"]
+    st = nexus.device_status(stream)
+    if st != nexus.OK:
+        raise RuntimeError(f"device status after the tool-scan timing: {nexus.status_string(st)}")
+    gbs = big_bytes / (big_us * 1e-6) / 1e9
+    out = {"kernel": "slb_kernel",
+           "paper_size": {"tools": 250, "dim": 768, "queries": 1, "kernel_us": small_us,
+                          "route_e2e_us_p50": float(np.median(t_e2e)) * 1e6,
+                          "e2e": "host embedding -> quantise -> copy in -> scan + gate -> "
+                                 "decision copied out, through the Python binding"},
+           "large": {"tools": n_big, "dim": dim, "queries_per_launch": 32, "kernel_us": big_us,
+                     "queries_per_s": 32 / (big_us * 1e-6), "by_batch": by_batch},
+           "roofline": {"bound": "hbm", "kernel": "slb_kernel (1M x 768 codes, 32 queries)",
+                        "achieved": gbs, "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                        "frac": gbs / peaks["hbm_gbs"], "peak_kind": f"copy, {peak_kind}",
+                        "traffic": None}}
+    del big, ws_big
+    if with_oracle:
+        import oracle
+        oc, os_ = oracle.slb_quantize(x)
+        qc, qs = oracle.slb_quantize(q[:20])
+        t0 = time.perf_counter()
+        for i in range(20):
+            oracle.slb_route(qc[i:i + 1], qs[i:i + 1], oc, os_)
+        dt = (time.perf_counter() - t0) / 20
+        out["cpu_baseline"] = {"value": dt * 1e6, "unit": "us per query", "cores": 1,
+                               "kind": "oracle",
+                               "sample": "NumPy oracle: one query against 250 x 768 codes"}
     return out
 
 

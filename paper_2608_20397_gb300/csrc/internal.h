@@ -174,6 +174,7 @@ struct SlbLaunch {
   float tau;
 };
 constexpr int kSlbMaxQueries = 32;
+constexpr int kSlbSmallQueries = 4;   // up to this many queries: the latency path
 cudaError_t launch_slb(const SlbLaunch& p, int grid, cudaStream_t stream);
 
 }  // namespace nexus

@@ -250,10 +250,13 @@ bool encode_2d_sw128(CUtensorMap* m, const void* base, uint64_t inner, uint64_t 
   return r == CUDA_SUCCESS;
 }
 
-// Tool scan: CTAs of 8 warps, about 64 tools per CTA, at most two waves.
+// Tool scan: CTAs of 8 warps. Few queries (the latency path): 8 tools per CTA,
+// one per warp, as long as that fits two waves. Batches: about 64 tools per CTA.
+// Either way at most two waves of CTAs.
 constexpr size_t kSlbPartOffset = 256;
-int slb_grid(int32_t n_tools, int32_t* per_out) {
-  int grid = static_cast<int>(std::min<int64_t>((n_tools + 63) / 64, 2 * num_sms()));
+int slb_grid(int32_t n_tools, int32_t n_queries, int32_t* per_out) {
+  const int64_t target = n_queries <= kSlbSmallQueries ? 8 : 64;
+  int grid = static_cast<int>(std::min<int64_t>((n_tools + target - 1) / target, 2 * num_sms()));
   grid = std::max(grid, 1);
   const int32_t per = (n_tools + grid - 1) / grid;
   if (per_out) *per_out = per;
@@ -654,7 +657,7 @@ nexus_status nexus_suffix_qkv(const nexus_kv_cache* cache, const int32_t* d_page
 
 size_t nexus_slb_workspace_size(int32_t n_tools) {
   if (n_tools < 1) return 0;
-  const int grid = slb_grid(n_tools, nullptr);
+  const int grid = std::max(slb_grid(n_tools, 1, nullptr), slb_grid(n_tools, kSlbMaxQueries, nullptr));
   return kSlbPartOffset + static_cast<size_t>(grid) * kSlbMaxQueries * 2 * (sizeof(float) + sizeof(int32_t));
 }
 
@@ -677,22 +680,24 @@ nexus_status nexus_slb_route(const int8_t* d_tools, const float* d_tool_scales, 
   if (n_queries == 0) return NEXUS_OK;
   if (!workspace || !aligned16(workspace) || workspace_bytes < nexus_slb_workspace_size(n_tools))
     return NEXUS_ENOMEM;
-  int32_t per = 0;
-  const int grid = slb_grid(n_tools, &per);
+  const int grid_max = std::max(slb_grid(n_tools, 1, nullptr),
+                                slb_grid(n_tools, kSlbMaxQueries, nullptr));
   uint8_t* ws = static_cast<uint8_t*>(workspace);
   SlbLaunch p;
   p.tools = d_tools;
   p.tool_scales = d_tool_scales;
   p.n_tools = n_tools;
   p.dim = dim;
-  p.tools_per_cta = per;
   p.tau = tau;
   p.counter = reinterpret_cast<unsigned int*>(ws);
   p.part_score = reinterpret_cast<float*>(ws + kSlbPartOffset);
   p.part_idx = reinterpret_cast<int32_t*>(ws + kSlbPartOffset +
-                                          static_cast<size_t>(grid) * kSlbMaxQueries * 2 * sizeof(float));
+                                          static_cast<size_t>(grid_max) * kSlbMaxQueries * 2 * sizeof(float));
   for (int32_t q0 = 0; q0 < n_queries; q0 += kSlbMaxQueries) {
     p.n_queries = std::min(kSlbMaxQueries, n_queries - q0);
+    int32_t per = 0;
+    const int grid = slb_grid(n_tools, p.n_queries, &per);
+    p.tools_per_cta = per;
     p.queries = d_queries + static_cast<int64_t>(q0) * dim;
     p.query_scales = d_query_scales + q0;
     p.top_idx = d_top_idx + 2 * static_cast<int64_t>(q0);

@@ -4,15 +4,18 @@
 // the two best tools (score, then lower index); routed to the best one when the
 // margin top1 - top2 exceeds tau, else escalated (-1).
 //
-// One warp scores one tool against every query of the launch (up to 32): lane l
-// reads 4-byte words l, l + 32, ... of the tool row (coalesced), multiplies them
-// with the same words of each query (shared memory) by dp4a, and a 31-shuffle
-// butterfly leaves lane q with the exact integer dot of query q. Lane q keeps
-// query q's running top two, so no further shuffles are needed. Warps merge in
-// shared memory, CTAs write their top two per query to the workspace, and the
-// CTA that finishes last (an atomic ticket; nothing waits) merges them, applies
-// the gate and resets the ticket for the next call. The merge uses a total order
-// (score, then index), so the result does not depend on the CTAs' timing.
+// One warp scores one tool at a time: lane l reads 4-byte words l, l + 32, ... of
+// the tool row (coalesced) and multiplies them with the same words of each query
+// by dp4a. Batches of 5..32 queries (slb_kernel) keep the queries in shared
+// memory and reduce with a 31-shuffle butterfly that leaves lane q with the exact
+// integer dot of query q, so lane q keeps query q's running top two. Up to 4
+// queries (slb_small_kernel, the routing of single requests) read the query
+// words straight into registers, load all of a tool's words at once and run
+// with one or two tools per warp, for latency. Warps merge in shared memory,
+// CTAs write their top two per query to the workspace, and the CTA that
+// finishes last (an atomic ticket; nothing waits) merges them, applies the gate
+// and resets the ticket for the next call. The merge uses a total order (score,
+// then index), so the result does not depend on the CTAs' timing.
 #include <cstdint>
 
 #include "internal.h"
@@ -48,6 +51,47 @@ __device__ __forceinline__ Top2 empty_top2() {
   return a;
 }
 
+__device__ __forceinline__ Top2 shfl_top2(const Top2& a, int off) {
+  Top2 b;
+  b.s1 = __shfl_xor_sync(0xffffffffu, a.s1, off);
+  b.s2 = __shfl_xor_sync(0xffffffffu, a.s2, off);
+  b.i1 = __shfl_xor_sync(0xffffffffu, a.i1, off);
+  b.i2 = __shfl_xor_sync(0xffffffffu, a.i2, off);
+  return b;
+}
+
+// Run by every thread of the CTA that finished last: warp w merges the CTA
+// partials of queries w, w + 8, ..., its lanes striding over the CTAs (their
+// loads are independent, so they overlap), then a shuffle merge of the lanes'
+// top twos; applies the gate and resets the ticket.
+__device__ void final_merge(const SlbLaunch& p, int warp, int lane) {
+  __threadfence();
+  for (int q = warp; q < p.n_queries; q += kSlbWarps) {
+    Top2 m = empty_top2();
+    for (int b = lane; b < (int)gridDim.x; b += 32) {
+      const int64_t k = (int64_t)b * 32 + q;
+      push(m, __ldcg(p.part_score + 2 * k), __ldcg(p.part_idx + 2 * k));
+      push(m, __ldcg(p.part_score + 2 * k + 1), __ldcg(p.part_idx + 2 * k + 1));
+    }
+#pragma unroll
+    for (int off = 16; off >= 1; off >>= 1) {
+      const Top2 o = shfl_top2(m, off);
+      push(m, o.s1, o.i1);
+      push(m, o.s2, o.i2);
+    }
+    if (lane == 0) {
+      const bool has2 = m.i2 != INT32_MAX;
+      const float s2 = has2 ? m.s2 : -INFINITY;
+      p.top_idx[2 * q] = m.i1;
+      p.top_idx[2 * q + 1] = has2 ? m.i2 : -1;
+      p.top_score[2 * q] = m.s1;
+      p.top_score[2 * q + 1] = s2;
+      p.route[q] = (m.s1 - s2) > p.tau ? m.i1 : -1;
+    }
+  }
+  if (threadIdx.x == 0) *p.counter = 0u;
+}
+
 template <int kQ>
 __global__ void __launch_bounds__(kSlbThreads) slb_kernel(const __grid_constant__ SlbLaunch p) {
   extern __shared__ int32_t s_q[];   // [kQ][words] query codes as 4-byte words
@@ -67,31 +111,53 @@ __global__ void __launch_bounds__(kSlbThreads) slb_kernel(const __grid_constant_
   Top2 top = empty_top2();
   const int t0 = blockIdx.x * p.tools_per_cta;
   const int t1 = min(p.n_tools, t0 + p.tools_per_cta);
-  for (int t = t0 + warp; t < t1; t += kSlbWarps) {
-    const int32_t* row = reinterpret_cast<const int32_t*>(p.tools + (int64_t)t * p.dim);
-    int acc[32];
+  // Two tools per step: each query word read from shared memory feeds two dp4a.
+  for (int ta = t0 + 2 * warp; ta < t1; ta += 2 * kSlbWarps) {
+    const bool has_b = ta + 1 < t1;
+    const int32_t* row_a = reinterpret_cast<const int32_t*>(p.tools + (int64_t)ta * p.dim);
+    const int32_t* row_b = row_a + (has_b ? words : 0);
+    int acc[2][32];
 #pragma unroll
-    for (int q = 0; q < 32; ++q) acc[q] = 0;
-    for (int w = lane; w < words; w += 32) {
-      const int32_t tw = __ldg(row + w);
+    for (int q = 0; q < 32; ++q) acc[0][q] = acc[1][q] = 0;
+    for (int w0 = lane; w0 < words; w0 += 32 * 8) {
+      int32_t wa[8], wb[8];
 #pragma unroll
-      for (int q = 0; q < kQ; ++q) acc[q] = __dp4a(tw, s_q[q * words + w], acc[q]);
+      for (int k = 0; k < 8; ++k) {
+        const int w = w0 + 32 * k;
+        wa[k] = w < words ? __ldg(row_a + w) : 0;
+        wb[k] = w < words ? __ldg(row_b + w) : 0;
+      }
+#pragma unroll
+      for (int k = 0; k < 8; ++k) {
+        const int w = w0 + 32 * k;
+        if (w >= words) break;
+#pragma unroll
+        for (int q = 0; q < kQ; ++q) {
+          const int32_t qw = s_q[q * words + w];
+          acc[0][q] = __dp4a(wa[k], qw, acc[0][q]);
+          acc[1][q] = __dp4a(wb[k], qw, acc[1][q]);
+        }
+      }
     }
-    // Butterfly: after the step of width `off`, lane bit b of `off` selects
-    // which half of the remaining queries this lane sums; lane l ends with query l.
 #pragma unroll
-    for (int off = 16; off >= 1; off >>= 1) {
-      const bool upper = (lane & off) != 0;
+    for (int x = 0; x < 2; ++x) {
+      // Butterfly: at the step of width `off`, this lane's bit `off` picks which
+      // half of the remaining queries it keeps summing; lane l ends with query l.
 #pragma unroll
-      for (int j = 0; j < off; ++j) {
-        const int send = upper ? acc[j] : acc[j + off];
-        const int keep = upper ? acc[j + off] : acc[j];
-        acc[j] = keep + __shfl_xor_sync(0xffffffffu, send, off);
+      for (int off = 16; off >= 1; off >>= 1) {
+        const bool upper = (lane & off) != 0;
+#pragma unroll
+        for (int j = 0; j < off; ++j) {
+          const int send = upper ? acc[x][j] : acc[x][j + off];
+          const int keep = upper ? acc[x][j + off] : acc[x][j];
+          acc[x][j] = keep + __shfl_xor_sync(0xffffffffu, send, off);
+        }
       }
     }
     if (lane < nq) {
-      const float c = qscale * __ldg(p.tool_scales + t);
-      push(top, __int2float_rn(acc[0]) * c, t);
+      push(top, __int2float_rn(acc[0][0]) * (qscale * __ldg(p.tool_scales + ta)), ta);
+      if (has_b)
+        push(top, __int2float_rn(acc[1][0]) * (qscale * __ldg(p.tool_scales + ta + 1)), ta + 1);
     }
   }
   s_top[warp][lane] = top;
@@ -115,24 +181,96 @@ __global__ void __launch_bounds__(kSlbThreads) slb_kernel(const __grid_constant_
   __syncthreads();
   if (threadIdx.x == 0) s_last = atomicAdd(p.counter, 1u) == gridDim.x - 1;
   __syncthreads();
-  if (!s_last || warp != 0) return;
-  __threadfence();
-  if (lane < nq) {
-    Top2 m = empty_top2();
-    for (int b = 0; b < (int)gridDim.x; ++b) {
-      const int64_t k = (int64_t)b * 32 + lane;
-      push(m, __ldcg(p.part_score + 2 * k), __ldcg(p.part_idx + 2 * k));
-      push(m, __ldcg(p.part_score + 2 * k + 1), __ldcg(p.part_idx + 2 * k + 1));
+  if (s_last) final_merge(p, warp, lane);
+}
+
+// Few queries (the routing of one request): the latency path. Query words are
+// read straight into registers (no shared-memory staging before the scan can
+// start), each warp takes one tool at a time with all of its words loaded at
+// once, and the host gives it enough CTAs that a warp sees one or two tools.
+template <int kQ, int kT>
+__global__ void __launch_bounds__(kSlbThreads) slb_small_kernel(const __grid_constant__ SlbLaunch p) {
+  __shared__ Top2 s_top[kSlbWarps][kQ];
+  __shared__ bool s_last;
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  const int words = p.dim / 4;
+  const int nq = p.n_queries;
+  const int32_t* qsrc = reinterpret_cast<const int32_t*>(p.queries);
+
+  Top2 top[kQ];
+#pragma unroll
+  for (int q = 0; q < kQ; ++q) top[q] = empty_top2();
+  const int t0 = blockIdx.x * p.tools_per_cta;
+  const int t1 = min(p.n_tools, t0 + p.tools_per_cta);
+  // kT tools per warp step, every word of the step loaded before any product.
+  for (int ta = t0 + kT * warp; ta < t1; ta += kT * kSlbWarps) {
+    int acc[kT][kQ];
+#pragma unroll
+    for (int x = 0; x < kT; ++x)
+#pragma unroll
+      for (int q = 0; q < kQ; ++q) acc[x][q] = 0;
+    for (int w0 = lane; w0 < words; w0 += 32 * 8) {
+      int32_t tw[kT][8];
+#pragma unroll
+      for (int x = 0; x < kT; ++x) {
+        const int32_t* row = reinterpret_cast<const int32_t*>(p.tools + (int64_t)(ta + x) * p.dim);
+#pragma unroll
+        for (int k = 0; k < 8; ++k) {
+          const int w = w0 + 32 * k;
+          tw[x][k] = (ta + x < t1 && w < words) ? __ldg(row + w) : 0;
+        }
+      }
+#pragma unroll
+      for (int q = 0; q < kQ; ++q) {
+#pragma unroll
+        for (int k = 0; k < 8; ++k) {
+          const int w = w0 + 32 * k;
+          const int32_t qw = (q < nq && w < words) ? __ldg(qsrc + q * words + w) : 0;
+#pragma unroll
+          for (int x = 0; x < kT; ++x) acc[x][q] = __dp4a(tw[x][k], qw, acc[x][q]);
+        }
+      }
     }
-    const bool has2 = m.i2 != INT32_MAX;
-    const float s2 = has2 ? m.s2 : -INFINITY;
-    p.top_idx[2 * lane] = m.i1;
-    p.top_idx[2 * lane + 1] = has2 ? m.i2 : -1;
-    p.top_score[2 * lane] = m.s1;
-    p.top_score[2 * lane + 1] = s2;
-    p.route[lane] = (m.s1 - s2) > p.tau ? m.i1 : -1;
+#pragma unroll
+    for (int x = 0; x < kT; ++x) {
+#pragma unroll
+      for (int q = 0; q < kQ; ++q) {
+#pragma unroll
+        for (int off = 16; off >= 1; off >>= 1)
+          acc[x][q] += __shfl_xor_sync(0xffffffffu, acc[x][q], off);
+        if (q < nq && ta + x < t1) {
+          const float c = __ldg(p.query_scales + q) * __ldg(p.tool_scales + ta + x);
+          push(top[q], __int2float_rn(acc[x][q]) * c, ta + x);
+        }
+      }
+    }
   }
-  if (lane == 0) *p.counter = 0u;
+  if (lane == 0) {
+#pragma unroll
+    for (int q = 0; q < kQ; ++q) s_top[warp][q] = top[q];
+  }
+  __syncthreads();
+  if (warp == 0) {
+    if (lane < nq) {
+      Top2 m = s_top[0][lane];
+      for (int w = 1; w < kSlbWarps; ++w) {
+        const Top2 o = s_top[w][lane];
+        push(m, o.s1, o.i1);
+        push(m, o.s2, o.i2);
+      }
+      const int64_t k = (int64_t)blockIdx.x * 32 + lane;
+      p.part_score[2 * k] = m.s1;
+      p.part_score[2 * k + 1] = m.s2;
+      p.part_idx[2 * k] = m.i1;
+      p.part_idx[2 * k + 1] = m.i2;
+    }
+    __threadfence();
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) s_last = atomicAdd(p.counter, 1u) == gridDim.x - 1;
+  __syncthreads();
+  if (s_last) final_merge(p, warp, lane);
 }
 
 template <int kQ>
@@ -151,8 +289,19 @@ cudaError_t launch_slb_as(const SlbLaunch& p, int grid, cudaStream_t stream) {
 
 cudaError_t launch_slb(const SlbLaunch& p, int grid, cudaStream_t stream) {
   if (p.n_queries <= 0 || grid <= 0) return cudaSuccess;
-  if (p.n_queries <= 1) return launch_slb_as<1>(p, grid, stream);
-  if (p.n_queries <= 4) return launch_slb_as<4>(p, grid, stream);
+  if (p.n_queries <= kSlbSmallQueries) {
+    // Many tools per warp: four per step for more loads in flight; otherwise one
+    // per warp, so a small registry spreads over every warp.
+    const bool tiled = p.tools_per_cta >= 4 * 2 * kSlbWarps;
+    if (p.n_queries == 1) {
+      if (tiled) slb_small_kernel<1, 4><<<(unsigned)grid, kSlbThreads, 0, stream>>>(p);
+      else slb_small_kernel<1, 1><<<(unsigned)grid, kSlbThreads, 0, stream>>>(p);
+    } else {
+      if (tiled) slb_small_kernel<kSlbSmallQueries, 4><<<(unsigned)grid, kSlbThreads, 0, stream>>>(p);
+      else slb_small_kernel<kSlbSmallQueries, 1><<<(unsigned)grid, kSlbThreads, 0, stream>>>(p);
+    }
+    return cudaGetLastError();
+  }
   if (p.n_queries <= 8) return launch_slb_as<8>(p, grid, stream);
   if (p.n_queries <= 16) return launch_slb_as<16>(p, grid, stream);
   return launch_slb_as<32>(p, grid, stream);
