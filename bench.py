@@ -315,6 +315,8 @@ def main():
                     help="run only this kernel of the step (small case for ncu captures)")
     ap.add_argument("--workload", choices=["c5", "c3"], default="c5",
                     help="workload of --profile runs (c3: token-innermost V cache)")
+    ap.add_argument("--tokens", type=int, default=0,
+                    help="--profile qkv: re-decode this many last tokens of the spliced cache")
     args = ap.parse_args()
 
     rank = int(os.environ.get("RANK", "0"))
@@ -458,7 +460,9 @@ def _profile_only(wl, args, stream):
         # of the spliced span (c3: 2192 tokens) or the whole context of the
         # re-prefill (c5: 32768 tokens).
         from paper_2608_20397_gb300.workloads import HIDDEN, qkv_weights, randn_bf16
-        if args.workload == "c3":
+        if args.tokens > 0:
+            qkv_kv, qkv_n, qkv_row = wl.T, args.tokens, 1
+        elif args.workload == "c3":
             qkv_kv, qkv_n, qkv_row = wl.T, wl.w.sessions[0].suffix_span, 1
         else:
             qkv_kv, qkv_n, qkv_row = wl.n_past, wl.n_past, 0
@@ -570,14 +574,21 @@ def _qkv_measure(wl, stream, peaks, peak_kind, with_oracle, warmup=3, reps=10):
             one(i)
         a = torch.cuda.Event(enable_timing=True)
         e = torch.cuda.Event(enable_timing=True)
+        # a fixed-length sleep holds the stream while the launches are enqueued,
+        # so short launches are timed without the host's submission gaps
+        torch.cuda.synchronize()
+        torch.cuda._sleep(4_000_000)
         a.record(stream)
+        t0 = time.perf_counter()
         for i in range(reps):
             one(i)
+        host_us = (time.perf_counter() - t0) / reps * 1e6
         e.record(stream)
         torch.cuda.synchronize()
         ms = a.elapsed_time(e) / reps
         flops = 2.0 * n * HIDDEN * n_heads * D
-        out[name] = {"tokens": n, "ms_per_launch": ms, "tflops": flops / (ms * 1e-3) / 1e12}
+        out[name] = {"tokens": n, "ms_per_launch": ms, "tflops": flops / (ms * 1e-3) / 1e12,
+                     "host_us_per_call": host_us}
     st = nexus.device_status(stream)
     if st != nexus.OK:
         raise RuntimeError(f"device status after the Q/K/V timing: {nexus.status_string(st)}")

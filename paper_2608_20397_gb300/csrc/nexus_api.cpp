@@ -250,13 +250,16 @@ bool encode_2d_sw128(CUtensorMap* m, const void* base, uint64_t inner, uint64_t 
   return r == CUDA_SUCCESS;
 }
 
-// Tool scan: CTAs of 8 warps. Few queries (the latency path): 8 tools per CTA,
-// one per warp, as long as that fits two waves. Batches: about 64 tools per CTA.
-// Either way at most two waves of CTAs.
+// Tool scan: CTAs of 8 warps. Few queries (the latency path, 64 registers, 4
+// CTAs per SM): 8 tools per CTA, one per warp, up to four CTAs per SM, so a
+// large registry keeps 32 warps of loads in flight on every SM. Batches (one
+// CTA per SM by registers): about 64 tools per CTA, at most two waves.
 constexpr size_t kSlbPartOffset = 256;
 int slb_grid(int32_t n_tools, int32_t n_queries, int32_t* per_out) {
-  const int64_t target = n_queries <= kSlbSmallQueries ? 8 : 64;
-  int grid = static_cast<int>(std::min<int64_t>((n_tools + target - 1) / target, 2 * num_sms()));
+  const bool small = n_queries <= kSlbSmallQueries;
+  const int64_t target = small ? 8 : 64;
+  int grid = static_cast<int>(std::min<int64_t>((n_tools + target - 1) / target,
+                                                (small ? 4 : 2) * num_sms()));
   grid = std::max(grid, 1);
   const int32_t per = (n_tools + grid - 1) / grid;
   if (per_out) *per_out = per;
