@@ -845,7 +845,7 @@ def _slb_measure(wl, stream, peaks, peak_kind, with_oracle, reps=200):
            "roofline": {"bound": "hbm", "kernel": "slb_small_kernel (1M x 768 codes, 1 query)",
                         "achieved": gbs, "peak": peaks["hbm_gbs"], "unit": "GB/s",
                         "frac": gbs / peaks["hbm_gbs"], "peak_kind": f"copy, {peak_kind}",
-                        "traffic": None}}
+                        "traffic": _profiled_traffic("slb_small_kernel")}}
     del big, ws_big
     if with_oracle:
         import oracle
