@@ -214,6 +214,28 @@ __device__ __forceinline__ float tanh_from_exp2(float x2) {
   return fmaf(-2.f, r, 1.f);
 }
 
+// S = Q K^T over one 128-key tile: 8 products along d, then S-full committed.
+// Descriptors come in formed; a k-step adds its byte offset / 16 to the
+// start-address field (no carry: shared memory lies below 256 KiB), so a product
+// costs one 64-bit add per operand to issue.
+__device__ __forceinline__ void issue_s(uint32_t t_s, uint64_t dq, uint64_t dk, uint32_t idesc,
+                                        uint32_t s_full) {
+#pragma unroll
+  for (int kk = 0; kk < D / 16; ++kk) {
+    const uint64_t o = static_cast<uint64_t>(((kk >> 2) * kHalf + (kk & 3) * 32) >> 4);
+    mma_bf16(t_s, dq + o, dk + o, idesc, kk > 0 ? 1u : 0u);
+  }
+  mma_commit(s_full);
+}
+
+// O += P V over one 128-key tile: P from TMEM (16 keys = 8 columns per step).
+__device__ __forceinline__ void issue_pv(uint32_t t_o, uint32_t t_s, uint64_t dv, uint64_t v_step,
+                                         uint32_t idesc, bool first) {
+#pragma unroll
+  for (int kk = 0; kk < BN / 16; ++kk)
+    mma_bf16_ts(t_o, t_s + kk * 8, dv + kk * v_step, idesc, (!first || kk > 0) ? 1u : 0u);
+}
+
 // kSoftcap: attention-logit soft-capping (Sec. V-B): the scaled score s becomes
 // cap * tanh(s / cap) before the softmax.
 template <bool kSoftcap>
@@ -356,32 +378,22 @@ attention_kernel(const __grid_constant__ AttnLaunch p, const __grid_constant__ A
     // ------------------------------------------------------ MMA issuer
     constexpr uint32_t idesc_qk = idesc_bf16_f32(BM, BN, false);
     const uint32_t idesc_pv = idesc_bf16_f32(BM, D, !vt);
-    auto issue_s = [&](int x, int st) {   // S_x = Q_x K^T
-      const uint32_t qa = sbase + OFF_Q + x * kTileBytes;
-      const uint32_t ka = sbase + OFF_K + st * kTileBytes;
-      const uint32_t t_s = tmem + TM_S + x * 128;
-#pragma unroll
-      for (int kk = 0; kk < D / 16; ++kk) {
-        const uint32_t off = (kk >> 2) * kHalf + (kk & 3) * 32;
-        mma_bf16(t_s, smem_desc(qa + off, 16, 1024, kSwizzle128B),
-                 smem_desc(ka + off, 16, 1024, kSwizzle128B), idesc_qk, kk > 0);
-      }
-      mma_commit(bar(B_SF + x));
-    };
-    auto issue_pv = [&](int x, int st, bool first) {   // O_x += P_x V
-      const uint32_t va = sbase + OFF_V + st * kTileBytes;
-      const uint32_t t_s = tmem + TM_S + x * 128;
-      const uint32_t t_o = tmem + TM_O + x * 128;
-#pragma unroll
-      for (int kk = 0; kk < BN / 16; ++kk) {
-        // row-major V: MN-major, 64-wide d halves 16 KiB apart (LBO), 8-key
-        // groups 1 KiB apart (SBO); token-innermost V: K-major pages of
-        // [128 d][16 keys], 8-row groups 256 B apart. P: 16 keys = 8 columns.
-        const uint64_t bdesc = vt ? smem_desc(va + kk * 4096, 16, 256, kSwizzle32B)
-                                  : smem_desc(va + kk * 2048, kHalf, 1024, kSwizzle128B);
-        mma_bf16_ts(t_o, t_s + kk * 8, bdesc, idesc_pv, (!first || kk > 0) ? 1u : 0u);
-      }
-    };
+    // Shared-memory descriptors are formed once per CTA; a k-step only adds its
+    // byte offset / 16 to the start-address field (no carry out of the field:
+    // shared memory lies below 256 KiB). Forming descriptors per product made
+    // the issuing thread too slow to keep the tensor core fed.
+    const uint64_t dq0 = smem_desc(sbase + OFF_Q, 16, 1024, kSwizzle128B);
+    const uint64_t dq1 = smem_desc(sbase + OFF_Q + kTileBytes, 16, 1024, kSwizzle128B);
+    const uint64_t dk0 = smem_desc(sbase + OFF_K, 16, 1024, kSwizzle128B);
+    const uint64_t dk1 = smem_desc(sbase + OFF_K + kTileBytes, 16, 1024, kSwizzle128B);
+    // row-major V: MN-major, 64-wide d halves 16 KiB apart (LBO), 8-key groups
+    // 1 KiB apart (SBO), 16 keys = 2 KiB per k-step; token-innermost V: K-major
+    // pages of [128 d][16 keys], 8-row groups 256 B apart, one 4 KiB page per step
+    const uint64_t dv0 = vt ? smem_desc(sbase + OFF_V, 16, 256, kSwizzle32B)
+                            : smem_desc(sbase + OFF_V, kHalf, 1024, kSwizzle128B);
+    const uint64_t dv1 = vt ? smem_desc(sbase + OFF_V + kTileBytes, 16, 256, kSwizzle32B)
+                            : smem_desc(sbase + OFF_V + kTileBytes, kHalf, 1024, kSwizzle128B);
+    const uint64_t v_step = vt ? (4096 >> 4) : (2048 >> 4);
     // Lanes 0-3 wait on different barriers at once (0 = none).
     auto wait4 = [&](uint32_t b0, uint32_t p0, uint32_t b1, uint32_t p1, uint32_t b2, uint32_t p2,
                      uint32_t b3, uint32_t p3) -> bool {
@@ -399,7 +411,8 @@ attention_kernel(const __grid_constant__ AttnLaunch p, const __grid_constant__ A
       ok = wait4(bar(B_Q), 0, bar(B_KF), 0, 0, 0, 0, 0);
       if (ok && lane == 0) {
         tc_fence_after();
-        for (int x = 0; x < n_q; ++x) issue_s(x, 0);
+        for (int x = 0; x < n_q; ++x)
+          issue_s(tmem + TM_S + x * 128, x ? dq1 : dq0, dk0, idesc_qk, bar(B_SF + x));
         mma_commit(bar(B_KE + 0));
       }
       __syncwarp();
@@ -417,10 +430,12 @@ attention_kernel(const __grid_constant__ AttnLaunch p, const __grid_constant__ A
           if (!ok) break;
           if (lane == 0) {
             tc_fence_after();
-            issue_pv(x, st, j == 0);
+            issue_pv(tmem + TM_O + x * 128, tmem + TM_S + x * 128, st ? dv1 : dv0, v_step,
+                     idesc_pv, j == 0);
             if (x == n_q - 1) mma_commit(bar(B_VE + st));
             if (more) {
-              issue_s(x, nst);
+              issue_s(tmem + TM_S + x * 128, x ? dq1 : dq0, nst ? dk1 : dk0, idesc_qk,
+                      bar(B_SF + x));
               if (x == n_q - 1) mma_commit(bar(B_KE + nst));
             } else {
               mma_commit(bar(B_OD + x));
