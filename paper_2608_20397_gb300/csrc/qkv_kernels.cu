@@ -160,6 +160,11 @@ qkv_kernel(const __grid_constant__ QkvLaunch p, const __grid_constant__ QkvMaps 
     // ------------------------------------------------------ MMA issuer
     if (lane == 0) {
       constexpr uint32_t idesc = idesc_bf16_f32(BM, BN, false);
+      // Descriptors of stage 0 formed once; a stage and a k-step only add their
+      // byte offset / 16 to the start-address field (no carry: shared memory
+      // lies below 256 KiB), keeping the issuing thread off the critical path.
+      const uint64_t da0 = smem_desc(sbase, 16, 1024, kSwizzle128B);
+      const uint64_t db0 = smem_desc(sbase + kABytes, 16, 1024, kSwizzle128B);
       int it = 0, acc_it = 0;
       bool ok = true;
       for (int t = blockIdx.x; t < p.total_tiles && ok; t += gridDim.x, ++acc_it) {
@@ -175,11 +180,10 @@ qkv_kernel(const __grid_constant__ QkvLaunch p, const __grid_constant__ QkvMaps 
           ok = mbar_wait(bar(B_FULL + st), (it / kStages) & 1, kBudgetNs, abort, gabort);
           if (!ok) { record_timeout(abort); break; }
           tc_fence_after();
-          const uint32_t a = sbase + st * kStageBytes;
+          const uint64_t so = static_cast<uint64_t>((st * kStageBytes) >> 4);
 #pragma unroll
           for (int kk = 0; kk < BK / 16; ++kk)
-            mma_bf16(d, smem_desc(a + kk * 32, 16, 1024, kSwizzle128B),
-                     smem_desc(a + kABytes + kk * 32, 16, 1024, kSwizzle128B), idesc,
+            mma_bf16(d, da0 + so + (kk * 32 >> 4), db0 + so + (kk * 32 >> 4), idesc,
                      (kb | kk) != 0 ? 1u : 0u);
           mma_commit(bar(B_EMPTY + st));
         }
