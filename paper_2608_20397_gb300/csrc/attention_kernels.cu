@@ -214,6 +214,37 @@ __device__ __forceinline__ float tanh_from_exp2(float x2) {
   return fmaf(-2.f, r, 1.f);
 }
 
+// Packed two-wide float32 arithmetic (one instruction for two lanes of work):
+// the softmax shares its SM sub-partitions with the thread issuing the tensor
+// core products, so every instruction it saves is an issue slot for that thread.
+__device__ __forceinline__ float2 ffma2(float2 a, float2 b, float2 c) {
+  float2 d;
+  asm("{\n"
+      " .reg .b64 ra, rb, rc, rd;\n"
+      " mov.b64 ra, {%2, %3};\n"
+      " mov.b64 rb, {%4, %5};\n"
+      " mov.b64 rc, {%6, %7};\n"
+      " fma.rn.f32x2 rd, ra, rb, rc;\n"
+      " mov.b64 {%0, %1}, rd;\n"
+      "}\n"
+      : "=f"(d.x), "=f"(d.y)
+      : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y), "f"(c.x), "f"(c.y));
+  return d;
+}
+__device__ __forceinline__ float2 fadd2(float2 a, float2 b) {
+  float2 d;
+  asm("{\n"
+      " .reg .b64 ra, rb, rd;\n"
+      " mov.b64 ra, {%2, %3};\n"
+      " mov.b64 rb, {%4, %5};\n"
+      " add.rn.f32x2 rd, ra, rb;\n"
+      " mov.b64 {%0, %1}, rd;\n"
+      "}\n"
+      : "=f"(d.x), "=f"(d.y)
+      : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y));
+  return d;
+}
+
 // S = Q K^T over one 128-key tile: 8 products along d, then S-full committed.
 // Descriptors come in formed; a k-step adds its byte offset / 16 to the
 // start-address field (no carry: shared memory lies below 256 KiB), so a product
@@ -515,22 +546,24 @@ attention_kernel(const __grid_constant__ AttnLaunch p, const __grid_constant__ A
         m_run = mxs;
       }
       const float neg_m = (m_run == -INFINITY) ? 0.f : -m_run;
-      float sum[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};   // eight short chains
+      float2 sum[4] = {{0.f, 0.f}, {0.f, 0.f}, {0.f, 0.f}, {0.f, 0.f}};   // four pair chains
+      const float2 sc2 = make_float2(sc, sc);
+      const float2 nm2 = make_float2(neg_m, neg_m);
 #pragma unroll
       for (int q = 0; q < 8; ++q) {
         uint32_t pk[8];
 #pragma unroll
         for (int e = 0; e < 16; e += 2) {
-          float a = fmaf(s[q * 16 + e], sc, neg_m), b = fmaf(s[q * 16 + e + 1], sc, neg_m);
+          float2 ab = ffma2(make_float2(s[q * 16 + e], s[q * 16 + e + 1]), sc2, nm2);
           if (((e >> 1) & 7) >= 8 - kPolyPairsPer8) {
-            a = exp2_poly(a);
-            b = exp2_poly(b);
+            ab.x = exp2_poly(ab.x);
+            ab.y = exp2_poly(ab.y);
           } else {
-            a = ex2_approx(a);
-            b = ex2_approx(b);
+            ab.x = ex2_approx(ab.x);
+            ab.y = ex2_approx(ab.y);
           }
-          sum[(e >> 1) & 7] += a + b;
-          pk[e / 2] = pack_bf16x2(a, b);
+          sum[(e >> 1) & 3] = fadd2(sum[(e >> 1) & 3], ab);
+          pk[e / 2] = pack_bf16x2(ab.x, ab.y);
         }
         tmem_st8(t_s + q * 8, pk);   // P over the first 64 columns of S
       }
@@ -547,8 +580,8 @@ attention_kernel(const __grid_constant__ AttnLaunch p, const __grid_constant__ A
         }
       }
       tmem_st_wait();
-      l_run = l_run * alpha + (((sum[0] + sum[1]) + (sum[2] + sum[3])) +
-                               ((sum[4] + sum[5]) + (sum[6] + sum[7])));
+      l_run = l_run * alpha + (((sum[0].x + sum[0].y) + (sum[1].x + sum[1].y)) +
+                               ((sum[2].x + sum[2].y) + (sum[3].x + sum[3].y)));
       tc_fence_before();
       mbar_arrive(bar(B_PF + x));
     }
