@@ -204,16 +204,6 @@ __device__ __forceinline__ void tmem_st8(uint32_t taddr, const uint32_t (&r)[8])
                : "memory");
 }
 
-// tanh(x) = 1 - 2 / (e^(2x) + 1), from the exponential and reciprocal units;
-// absolute error about 4e-7, so a soft-capped logit cap * tanh(s / cap) errs by
-// ~4e-7 * cap (saturates correctly to +-1 for large |x|). `x2` is 2 x log2(e).
-__device__ __forceinline__ float tanh_from_exp2(float x2) {
-  const float e = ex2_approx(x2);
-  float r;
-  asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(r) : "f"(e + 1.f));
-  return fmaf(-2.f, r, 1.f);
-}
-
 // Packed two-wide float32 arithmetic (one instruction for two lanes of work):
 // the softmax shares its SM sub-partitions with the thread issuing the tensor
 // core products, so every instruction it saves is an issue slot for that thread.
@@ -243,6 +233,25 @@ __device__ __forceinline__ float2 fadd2(float2 a, float2 b) {
       : "=f"(d.x), "=f"(d.y)
       : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y));
   return d;
+}
+
+__device__ __forceinline__ float2 fmul2(float2 a, float2 b) {
+  float2 d;
+  asm("{\n"
+      " .reg .b64 ra, rb, rd;\n"
+      " mov.b64 ra, {%2, %3};\n"
+      " mov.b64 rb, {%4, %5};\n"
+      " mul.rn.f32x2 rd, ra, rb;\n"
+      " mov.b64 {%0, %1}, rd;\n"
+      "}\n"
+      : "=f"(d.x), "=f"(d.y)
+      : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y));
+  return d;
+}
+__device__ __forceinline__ float rcp_approx(float x) {
+  float r;
+  asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(r) : "f"(x));
+  return r;
 }
 
 // S = Q K^T over one 128-key tile: 8 products along d, then S-full committed.
@@ -516,8 +525,22 @@ attention_kernel(const __grid_constant__ AttnLaunch p, const __grid_constant__ A
           for (int e = 0; e < 32; ++e) s[q * 32 + e] = __uint_as_float(v[q][e]);
       }
       if constexpr (kSoftcap) {
+        // tanh(x) = 1 - 2 / (2^(2x log2 e) + 1) on pairs: the scaling, the +1 and
+        // the final 1 - 2r on the packed float32 pipe, ex2 and rcp on MUFU
+        const float2 ci = make_float2(p.softcap_in, p.softcap_in);
+        const float2 one = make_float2(1.f, 1.f), m2 = make_float2(-2.f, -2.f);
 #pragma unroll
-        for (int c = 0; c < BN; ++c) s[c] = tanh_from_exp2(s[c] * p.softcap_in);
+        for (int c = 0; c < BN; c += 2) {
+          float2 e = fmul2(make_float2(s[c], s[c + 1]), ci);
+          e.x = ex2_approx(e.x);
+          e.y = ex2_approx(e.y);
+          e = fadd2(e, one);
+          e.x = rcp_approx(e.x);
+          e.y = rcp_approx(e.y);
+          e = ffma2(m2, e, one);
+          s[c] = e.x;
+          s[c + 1] = e.y;
+        }
       }
       const int lim = pos_r - (w.kt_begin + j) * BN;   // keys c <= lim are visible
       if (lim < BN - 1) {
