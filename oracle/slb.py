@@ -53,9 +53,11 @@ def slb_quantize(x) -> Tuple[np.ndarray, np.ndarray]:
 
 def slb_scores(q_codes, q_scales, t_codes, t_scales) -> np.ndarray:
     """float32 scores [n_queries][n_tools] of the rule above."""
-    qc = np.asarray(q_codes, dtype=np.int64)
-    tc = np.asarray(t_codes, dtype=np.int64)
-    dots = qc @ tc.T                                   # exact integer dot products
+    # Integer dot products: every product and partial sum is an integer below
+    # 2^24, so a float64 matrix product computes them exactly.
+    qc = np.asarray(q_codes, dtype=np.float64)
+    tc = np.asarray(t_codes, dtype=np.float64)
+    dots = qc @ tc.T
     c = (np.asarray(q_scales, dtype=np.float32)[:, None] *
          np.asarray(t_scales, dtype=np.float32)[None, :])   # float32 products of the scales
     return dots.astype(np.float32) * c
