@@ -222,3 +222,17 @@ def test_qkv_bad_page_is_skipped_and_reported(dev):
     assert torch.equal(gk[16:].view(torch.int16),
                        c.k0[c.layer][torch.as_tensor(c.h_pt[0, 3], device=dev)].permute(1, 0, 2)
                        .reshape(16, 8, 128).view(torch.int16))
+
+
+def test_qkv_bench_size_32768_tokens_sampled(dev):
+    # The bench's launch: all 32768 tokens of the c5 re-prefill, one layer, hidden
+    # 5120, 40 + 8 + 8 heads; 256 sampled rows (every tile row position class and
+    # the ragged ends) against the oracle, and no write outside the cache slots.
+    c = QkvCase(dev, [32768], [32768], HIDDEN, seed=22, n_layers=1, layer=0)
+    c.run()
+    torch.cuda.synchronize()
+    r = np.random.default_rng(1)
+    rows = np.sort(np.unique(np.concatenate([r.choice(32768, 250, replace=False),
+                                             [0, 1, 127, 128, 32767, 32640]])))
+    c.check(rows=rows, what="32768 tokens")
+    c.check_untouched()

@@ -111,3 +111,28 @@ def test_slb_large_registry_and_workspace_reuse(dev):
     for a, b in zip(first, second):
         assert np.array_equal(a, b)
     assert not ws[:16].any()                        # the ticket is back at zero
+
+
+def test_slb_bench_size_one_million_tools(dev):
+    # The bench's large scan: 2^20 tools x 768 codes, one query and a batch of 32;
+    # the oracle scores in chunks (exact integers times float32 scales) and the
+    # top two are taken over all of them by the same ordering.
+    r = np.random.default_rng(30)
+    n = 1 << 20
+    tc = r.integers(-127, 128, (n, 768), dtype=np.int8)
+    ts = (r.random(n, dtype=np.float32) * np.float32(0.01)).astype(np.float32)
+    qc = r.integers(-127, 128, (32, 768), dtype=np.int8)
+    qs = (r.random(32, dtype=np.float32) * np.float32(0.01)).astype(np.float32)
+    # plant near-ties: tool 5 copies tool 7 (equal scores when scales match)
+    tc[5] = tc[7]
+    ts[5] = ts[7]
+    for nq in (1, 32):
+        top_idx, top_score, route = run(dev, tc, ts, qc[:nq], qs[:nq])
+        scores = np.concatenate([oracle.slb_scores(qc[:nq], qs[:nq], tc[i:i + 65536], ts[i:i + 65536])
+                                 for i in range(0, n, 65536)], axis=1)
+        for a in range(nq):
+            order = np.lexsort((np.arange(n), -scores[a].astype(np.float64)))[:2]   # score, then index
+            (i1, s1), (i2, s2) = [(int(j), scores[a, j]) for j in order]
+            assert (top_idx[a, 0], top_idx[a, 1]) == (i1, i2), (nq, a)
+            assert top_score[a, 0] == s1 and top_score[a, 1] == s2
+            assert route[a] == (i1 if np.float32(s1 - s2) > np.float32(TAU) else -1)

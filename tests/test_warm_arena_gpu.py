@@ -142,3 +142,50 @@ def test_warm_start_attention_equals_cold(dev):
     assert same_bits(outs[0][0], outs[1][0])
     assert torch.equal(outs[0][1], outs[1][1])
     assert torch.isfinite(outs[0][0].float()).all()
+
+
+def test_warm_forks_at_bench_shape(dev):
+    """The bench's arena shape: 48 layers x 8 KV heads, 32 slots holding a shared
+    8192-token prompt and a 1024-token tail each; forks of 8192 + k tokens get
+    rows bit-identical to the slot's, through one copied boundary page."""
+    Lb, H = 48, 8
+    n_pages = 512 + 32 * 64 + 64
+    kp = torch.zeros((Lb, n_pages, H, PAGE, D), dtype=torch.bfloat16, device=dev)
+    vp = torch.zeros_like(kp)
+    cache = nexus.kv_cache(kp, vp, n_pages, Lb, H)
+    pool = nexus.PagePool(n_pages)
+    arena = nexus.WarmArena(32, 8192 + 1024)
+    r = np.random.default_rng(77)
+    system = [int(t) for t in r.integers(0, 32000, 8192)]
+    sys_pt = pool.alloc(512)
+    g = torch.Generator(device=dev)
+    g.manual_seed(5)
+    kp[:, torch.as_tensor(sys_pt, device=dev).long()] = torch.randn(
+        (Lb, 512, H, PAGE, D), generator=g, device=dev).to(torch.bfloat16)
+    tails = []
+    for s in range(32):
+        tail = [int(t) for t in r.integers(0, 32000, 1024)]
+        tails.append(tail)
+        own = pool.alloc(64)
+        kp[:, torch.as_tensor(own, device=dev).long()] = torch.randn(
+            (Lb, 64, H, PAGE, D), generator=g, device=dev).to(torch.bfloat16)
+        vp[:, torch.as_tensor(own, device=dev).long()] = -kp[:, torch.as_tensor(own, device=dev).long()]
+        pt = np.concatenate([sys_pt, own]).astype(np.int32)
+        pool.retain(sys_pt)
+        arena.store(pool, system + tail, pt)
+        pool.free(pt)
+    pool.free(sys_pt)
+    for j, k in ((0, 1), (7, 500), (31, 1023), (12, 16)):
+        q = system + tails[j][:k] + [40000 + i for i in range(64)]
+        slot, m = arena.match(q)
+        assert m == 8192 + k
+        pre, src, dst = arena.fork(pool, slot, m, -(-len(q) // PAGE))
+        nexus.copy_pages(cache, src, dst, 0, Lb)
+        torch.cuda.synchronize()
+        _, spages = arena.slot(slot)
+        gk, gv = read(kp, vp, pre, m)
+        wk, wv = read(kp, vp, spages, m)
+        assert same_bits(gk, wk) and same_bits(gv, wv)
+        pool.free(pre)
+    arena.close(pool)
+    assert pool.available() == n_pages
