@@ -517,6 +517,9 @@ def _profile_only(wl, args, stream):
     torch.cuda.synchronize()
     a = torch.cuda.Event(enable_timing=True)
     b = torch.cuda.Event(enable_timing=True)
+    # a fixed-length sleep holds the stream while the launches are enqueued, so
+    # short launches are timed without the host's submission gaps
+    torch.cuda._sleep(4_000_000)
     a.record(stream)
     for _ in range(args.steps):
         one()
