@@ -890,21 +890,23 @@ def _e2e(wl, stream, args, barrier, world, dist, dev):
     import torch
     L = wl.L
     nexus = wl.nexus
-    h_bk = torch.empty(wl.bk.shape, dtype=torch.bfloat16, pin_memory=True)
-    h_bv = torch.empty(wl.bv.shape, dtype=torch.bfloat16, pin_memory=True)
+    # Host buffers in the library's registered staging memory (nexus_host_alloc):
+    # on Grace hosts some cudaHostAlloc'd buffers copy at a tenth of the link rate.
+    host = lambda t: nexus.host_empty(t.shape, t.dtype)
+    h_bk, h_bv = host(wl.bk), host(wl.bv)
     h_bk.copy_(wl.bk)
     h_bv.copy_(wl.bv)
-    h_q = torch.empty(wl.q_pre.shape, dtype=torch.bfloat16, pin_memory=True)   # every layer's Q
-    h_o = torch.empty((2,) + tuple(wl.o_pre.shape[1:]), dtype=torch.bfloat16, pin_memory=True)
-    h_qs = torch.empty(wl.q_suf.shape, dtype=torch.bfloat16, pin_memory=True)
-    h_os = torch.empty(wl.o_suf.shape, dtype=torch.bfloat16, pin_memory=True)
-    h_q.copy_(wl.q_pre)
+    h_q = [host(wl.q_pre[l]) for l in range(L)]            # one buffer per layer's Q
+    h_o = [host(wl.o_pre[0]) for _ in range(2)]
+    h_qs, h_os = host(wl.q_suf), host(wl.o_suf)
+    for l in range(L):
+        h_q[l].copy_(wl.q_pre[l])
     h_qs.copy_(wl.q_suf)
     qbuf = [torch.empty_like(wl.q_pre[:1]) for _ in range(2)]
     obuf = [torch.empty_like(wl.o_pre[:1]) for _ in range(2)]
     s_in = torch.cuda.Stream(device=dev)
     s_out = torch.cuda.Stream(device=dev)
-    h2d = (h_bk.numel() + h_bv.numel() + h_q.numel() + h_qs.numel()) * 2
+    h2d = (h_bk.numel() + h_bv.numel() + sum(x.numel() for x in h_q) + h_qs.numel()) * 2
     d2h = (L * h_o[0].numel() + h_os.numel()) * 2
     ev = lambda: torch.cuda.Event()
 

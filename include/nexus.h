@@ -31,6 +31,9 @@
  *                            (Sec. V-D)
  *   nexus_slb_*              INT8 tool scan with the top-2 margin gate of the
  *                            semantic lookaside buffer (Sec. IV-A)
+ *   nexus_host_alloc, nexus_host_free
+ *                            page-locked host staging memory for the copies
+ *                            around the path
  *
  * Conventions
  *   - Device buffers are owned by the caller. The library never allocates or
@@ -491,6 +494,27 @@ nexus_status nexus_suffix_attention_noalloc(const nexus_kv_cache* cache,
                                             float* lse, int32_t n_q_heads, int32_t layer_begin,
                                             int32_t layer_end, int32_t split_kv,
                                             nexus_stream stream);
+
+/* ------------------------------------------------------ host staging memory */
+/* Page-locked host memory for the host<->device copies around the path (the
+ * per-layer Q/O transfers of a re-prefill, a compiled block read from host
+ * memory). The paper has no counterpart; this is a deployment convenience of
+ * this library. The library maps `bytes` (rounded up to the host page size) of
+ * fresh anonymous memory and registers it with the CUDA driver, so
+ * cudaMemcpyAsync from or to it is asynchronous and runs at the link rate.
+ * Grace hosts were seen to copy from some page-locked buffers made by
+ * cudaHostAlloc at a tenth of the rate of others; registered anonymous pages
+ * copied at one steady rate.
+ *
+ * *out receives the page-aligned address (zero-filled memory) or NULL.
+ * NEXUS_EINVAL for bytes == 0 or out == NULL, NEXUS_ENOMEM if the mapping
+ * fails, NEXUS_ECUDA if the driver refuses the registration (no GPU, or the
+ * page-locked limit is reached); nothing is left mapped on failure. The caller
+ * owns the memory and returns it with nexus_host_free, giving the same size. */
+nexus_status nexus_host_alloc(size_t bytes, void** out);
+/* Unregisters and unmaps memory from nexus_host_alloc. No copy may still be
+ * reading or writing it. NULL is a no-op; NEXUS_EINVAL for bytes == 0. */
+nexus_status nexus_host_free(void* p, size_t bytes);
 
 #ifdef __cplusplus
 }

@@ -4,6 +4,8 @@
 #include <cuda.h>
 #include <cudaTypedefs.h>
 #include <cuda_runtime.h>
+#include <sys/mman.h>
+#include <unistd.h>
 
 #include <algorithm>
 #include <cmath>
@@ -735,6 +737,38 @@ nexus_status nexus_slb_quantize(const float* h_x, int32_t n, int32_t dim, int8_t
     h_scales[i] = scale;
   }
   return NEXUS_OK;
+}
+
+// Page-locked staging memory: fresh anonymous pages registered with the driver.
+static size_t host_mapping_len(size_t bytes) {
+  const long pg = sysconf(_SC_PAGESIZE);
+  const size_t page = pg > 0 ? static_cast<size_t>(pg) : 4096;
+  return (bytes + page - 1) / page * page;
+}
+
+nexus_status nexus_host_alloc(size_t bytes, void** out) {
+  if (!out) return NEXUS_EINVAL;
+  *out = nullptr;
+  if (bytes == 0 || bytes > (static_cast<size_t>(1) << 48)) return NEXUS_EINVAL;
+  const size_t len = host_mapping_len(bytes);
+  void* p = mmap(nullptr, len, PROT_READ | PROT_WRITE, MAP_PRIVATE | MAP_ANONYMOUS, -1, 0);
+  if (p == MAP_FAILED) return NEXUS_ENOMEM;
+  if (cudaHostRegister(p, len, cudaHostRegisterDefault) != cudaSuccess) {
+    cudaGetLastError();
+    munmap(p, len);
+    return NEXUS_ECUDA;
+  }
+  *out = p;
+  return NEXUS_OK;
+}
+
+nexus_status nexus_host_free(void* p, size_t bytes) {
+  if (!p) return NEXUS_OK;
+  if (bytes == 0) return NEXUS_EINVAL;
+  const bool unregistered = cudaHostUnregister(p) == cudaSuccess;
+  if (!unregistered) cudaGetLastError();
+  munmap(p, host_mapping_len(bytes));
+  return unregistered ? NEXUS_OK : NEXUS_ECUDA;
 }
 
 size_t nexus_attention_workspace_size(int32_t n_seqs, const int32_t* h_kv_len,

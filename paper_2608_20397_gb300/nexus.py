@@ -134,6 +134,8 @@ _SIGS = {
     "nexus_suffix_qkv": (c_int32, [POINTER(KvCache), c_void_p, _i32p, c_int32, c_int32, c_int32,
                                    _i32p, _i32p, _i32p, c_void_p, c_int32, c_void_p, c_void_p,
                                    c_int32, c_int32, c_void_p, c_void_p]),
+    "nexus_host_alloc": (c_int32, [c_size_t, POINTER(c_void_p)]),
+    "nexus_host_free": (c_int32, [c_void_p, c_size_t]),
 }
 EXPORTED = tuple(_SIGS)
 
@@ -540,3 +542,34 @@ def slb_route(tools, tool_scales, queries, query_scales, top_idx, top_score, rou
         _ptr(tools), _ptr(tool_scales), int(tools.shape[0]), int(tools.shape[1]), _ptr(queries),
         _ptr(query_scales), int(queries.shape[0]), float(tau), _ptr(top_idx), _ptr(top_score),
         _ptr(route), _ptr(workspace), int(workspace.numel()), _stream(stream)))
+
+
+# ---------------------------------------------------- host staging memory
+class _HostMapping:
+    """Owns one nexus_host_alloc mapping; freed when the last tensor viewing it
+    is gone."""
+
+    def __init__(self, nbytes: int):
+        p = c_void_p()
+        _check("nexus_host_alloc", lib().nexus_host_alloc(int(nbytes), ctypes.byref(p)))
+        self.ptr, self.nbytes = int(p.value), int(nbytes)
+
+    def __del__(self):
+        if self.ptr and _lib is not None:
+            _lib.nexus_host_free(c_void_p(self.ptr), c_size_t(self.nbytes))
+            self.ptr = 0
+
+
+def host_empty(shape, dtype):
+    """A CPU torch tensor of ``shape`` / ``dtype`` (zero-filled) in page-locked
+    staging memory from nexus_host_alloc: copies between it and the device with
+    ``non_blocking=True`` are asynchronous (torch's ``is_pinned()`` reports only
+    its own allocator's memory and says False here). The memory is returned when
+    the tensor and every view of it are gone."""
+    import torch
+    shape = tuple(int(n) for n in shape)
+    nbytes = int(np.prod(shape, dtype=np.int64)) * torch.empty((), dtype=dtype).element_size()
+    m = _HostMapping(max(nbytes, 1))
+    raw = (ctypes.c_char * max(nbytes, 1)).from_address(m.ptr)
+    raw._mapping = m                        # the tensor's storage keeps `raw`, and so `m`, alive
+    return torch.frombuffer(raw, dtype=torch.uint8)[:nbytes].view(dtype).view(shape)

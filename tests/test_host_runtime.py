@@ -383,3 +383,18 @@ def test_slb_route_argument_checks():
     assert call(ws_bytes=ws - 1) == nexus.ENOMEM
     assert call(wsp=None) == nexus.ENOMEM
     assert call(nq=0) == nexus.OK                # nothing to scan: no launch
+
+
+def test_host_staging_argument_checks():
+    L = nexus.lib()
+    out = ctypes.c_void_p(1234)
+    assert L.nexus_host_alloc(0, ctypes.byref(out)) == nexus.EINVAL and not out.value
+    assert L.nexus_host_alloc(4096, None) == nexus.EINVAL
+    assert L.nexus_host_alloc(1 << 60, ctypes.byref(out)) == nexus.EINVAL
+    assert L.nexus_host_free(None, 4096) == nexus.OK
+    import torch
+    if not torch.cuda.is_available():
+        # no driver to register with: nothing is left mapped and NULL comes back
+        assert L.nexus_host_alloc(1 << 20, ctypes.byref(out)) == nexus.ECUDA and not out.value
+        with pytest.raises(nexus.NexusError):
+            nexus.host_empty((4, 4), torch.bfloat16)

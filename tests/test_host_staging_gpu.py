@@ -1,0 +1,54 @@
+"""Page-locked staging memory from nexus_host_alloc: registered with the
+driver, zero-filled, and asynchronous copies to and from it move the bytes
+unchanged."""
+import ctypes
+
+import pytest
+import torch
+
+from paper_2608_20397_gb300 import nexus
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def dev():
+    if not torch.cuda.is_available():
+        pytest.skip("no GPU")
+    return torch.device("cuda:0")
+
+
+@pytest.mark.parametrize("shape", [(1,), (3, 1000), (48, 65536 + 7), (2, 1 << 22)])
+def test_round_trip_through_staging(dev, shape):
+    h_in = nexus.host_empty(shape, torch.bfloat16)
+    h_out = nexus.host_empty(shape, torch.bfloat16)
+    assert not h_in.view(torch.int16).any()                 # fresh pages are zero
+    g = torch.Generator().manual_seed(1)
+    h_in.copy_(torch.randn(shape, generator=g).to(torch.bfloat16))
+    s = torch.cuda.Stream(device=dev)
+    d = torch.empty(shape, dtype=torch.bfloat16, device=dev)
+    with torch.cuda.stream(s):
+        d.copy_(h_in, non_blocking=True)
+        d.mul_(-1)
+        h_out.copy_(d, non_blocking=True)
+    s.synchronize()
+    assert torch.equal(h_out.view(torch.int16), (-h_in).view(torch.int16))
+
+
+def test_direct_alloc_and_free(dev):
+    L = nexus.lib()
+    p = ctypes.c_void_p()
+    assert L.nexus_host_alloc(5000, ctypes.byref(p)) == nexus.OK and p.value
+    assert p.value % 4096 == 0
+    ctypes.memset(p.value, 7, 5000)
+    assert L.nexus_host_free(p, 5000) == nexus.OK
+
+
+def test_views_keep_the_mapping(dev):
+    t = nexus.host_empty((1024, 128), torch.float32)
+    v = t[10:20]
+    del t
+    v.fill_(2.5)
+    d = v.to(dev, non_blocking=True)
+    torch.cuda.synchronize()
+    assert torch.equal(d.cpu(), torch.full((10, 128), 2.5))
