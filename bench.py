@@ -890,17 +890,19 @@ def _e2e(wl, stream, args, barrier, world, dist, dev):
     import torch
     L = wl.L
     nexus = wl.nexus
-    # Host buffers in the library's registered staging memory (nexus_host_alloc):
-    # on Grace hosts some cudaHostAlloc'd buffers copy at a tenth of the link rate.
-    host = lambda t: nexus.host_empty(t.shape, t.dtype)
-    h_bk, h_bv = host(wl.bk), host(wl.bv)
+    # Host buffers in the library's page-locked staging memory (nexus_host_alloc,
+    # huge pages where the request is large): every layer's Q in one region, the
+    # two O buffers in another.
+    host = lambda shape, dtype=torch.bfloat16: nexus.host_empty(shape, dtype)
+    h_bk, h_bv = host(wl.bk.shape), host(wl.bv.shape)
     h_bk.copy_(wl.bk)
     h_bv.copy_(wl.bv)
-    h_q = [host(wl.q_pre[l]) for l in range(L)]            # one buffer per layer's Q
-    h_o = [host(wl.o_pre[0]) for _ in range(2)]
-    h_qs, h_os = host(wl.q_suf), host(wl.o_suf)
-    for l in range(L):
-        h_q[l].copy_(wl.q_pre[l])
+    h_qall = host(wl.q_pre.shape)
+    h_q = [h_qall[l] for l in range(L)]
+    h_oall = host((2,) + tuple(wl.o_pre.shape[1:]))
+    h_o = [h_oall[0], h_oall[1]]
+    h_qs, h_os = host(wl.q_suf.shape), host(wl.o_suf.shape)
+    h_qall.copy_(wl.q_pre)
     h_qs.copy_(wl.q_suf)
     qbuf = [torch.empty_like(wl.q_pre[:1]) for _ in range(2)]
     obuf = [torch.empty_like(wl.o_pre[:1]) for _ in range(2)]

@@ -547,59 +547,77 @@ attention_kernel(const __grid_constant__ AttnLaunch p, const __grid_constant__ A
 #pragma unroll
         for (int c = 0; c < BN; ++c) s[c] = (c <= lim) ? s[c] : -INFINITY;
       }
-      // Row max as eight independent 3-input chains, then a short tree.
+      // One pass over the row: exponentials 2^(s sc - m) written to TMEM as
+      // bf16 P over the first 64 columns of S, four pair chains of the row sum,
+      // and, when `track`, the row max alongside (eight 3-input chains).
+      float2 sum[4];
       float mxa[8];
+      auto pass = [&](float neg_m, bool track) {
+        const float2 sc2 = make_float2(sc, sc);
+        const float2 nm2 = make_float2(neg_m, neg_m);
 #pragma unroll
-      for (int k = 0; k < 8; ++k) mxa[k] = fmax3(s[k], s[8 + k], s[16 + k]);
+        for (int k = 0; k < 4; ++k) sum[k] = make_float2(0.f, 0.f);
 #pragma unroll
-      for (int c = 24; c + 16 <= BN; c += 16)
+        for (int q = 0; q < 8; ++q) {
+          uint32_t pk[8];
 #pragma unroll
-        for (int k = 0; k < 8; ++k) mxa[k] = fmax3(mxa[k], s[c + k], s[c + 8 + k]);
-#pragma unroll
-      for (int k = 0; k < 8; ++k) mxa[k] = fmaxf(mxa[k], s[BN - 8 + k]);
-      const float mx = fmaxf(fmax3(mxa[0], mxa[1], mxa[2]),
-                             fmaxf(fmax3(mxa[3], mxa[4], mxa[5]), fmaxf(mxa[6], mxa[7])));
-      const float mxs = mx * sc;
-      // Move the running max only when the new one is far above it; the
-      // stale max keeps every p <= 2^8 and O / l unchanged.
-      float alpha = 1.f;
-      bool rescale = false;
-      if (mx > -INFINITY && (m_run == -INFINITY || mxs > m_run + kRescaleThreshold)) {
-        if (m_run != -INFINITY) { alpha = ex2_approx(m_run - mxs); rescale = true; }
-        m_run = mxs;
-      }
-      const float neg_m = (m_run == -INFINITY) ? 0.f : -m_run;
-      float2 sum[4] = {{0.f, 0.f}, {0.f, 0.f}, {0.f, 0.f}, {0.f, 0.f}};   // four pair chains
-      const float2 sc2 = make_float2(sc, sc);
-      const float2 nm2 = make_float2(neg_m, neg_m);
-#pragma unroll
-      for (int q = 0; q < 8; ++q) {
-        uint32_t pk[8];
-#pragma unroll
-        for (int e = 0; e < 16; e += 2) {
-          float2 ab = ffma2(make_float2(s[q * 16 + e], s[q * 16 + e + 1]), sc2, nm2);
-          if (((e >> 1) & 7) >= 8 - kPolyPairsPer8) {
-            ab.x = exp2_poly(ab.x);
-            ab.y = exp2_poly(ab.y);
-          } else {
+          for (int e = 0; e < 16; e += 2) {
+            const int c = q * 16 + e;
+            if (track) mxa[e >> 1] = fmax3(mxa[e >> 1], s[c], s[c + 1]);
+            float2 ab = ffma2(make_float2(s[c], s[c + 1]), sc2, nm2);
             ab.x = ex2_approx(ab.x);
             ab.y = ex2_approx(ab.y);
+            sum[(e >> 1) & 3] = fadd2(sum[(e >> 1) & 3], ab);
+            pk[e / 2] = pack_bf16x2(ab.x, ab.y);
           }
-          sum[(e >> 1) & 3] = fadd2(sum[(e >> 1) & 3], ab);
-          pk[e / 2] = pack_bf16x2(ab.x, ab.y);
+          tmem_st8(t_s + q * 8, pk);   // P over the first 64 columns of S
         }
-        tmem_st8(t_s + q * 8, pk);   // P over the first 64 columns of S
-      }
-      if (__any_sync(0xffffffffu, rescale)) {
-        // PV_x(j-1) is complete: this step's S-full barrier was committed after it.
-#pragma unroll 1
-        for (int q = 0; q < 4; ++q) {
-          uint32_t v[32];
-          tmem_ld32(t_o + q * 32, v);
-          tmem_ld_wait();
+      };
+      auto row_max = [&]() -> float {
+        return fmaxf(fmax3(mxa[0], mxa[1], mxa[2]),
+                     fmaxf(fmax3(mxa[3], mxa[4], mxa[5]), fmaxf(mxa[6], mxa[7])));
+      };
 #pragma unroll
-          for (int e = 0; e < 32; ++e) v[e] = __float_as_uint(__uint_as_float(v[e]) * alpha);
-          tmem_st32(t_o + q * 32, v);
+      for (int k = 0; k < 8; ++k) mxa[k] = -INFINITY;
+      // The running max moves only when a tile's max exceeds it by more than
+      // 2^8, which after a row's first tile is rare. So once every row of the
+      // warp has a running max, the exponentials are taken with it straight
+      // away and the tile's max is tracked alongside; only if it has grown past
+      // the threshold is the pass redone with the new max. Either way the
+      // result is that of taking the max first.
+      // (Soft-capped scores always take the max first: the tracked pass holds
+      // too many registers beside the capping arithmetic.)
+      const bool have_max = !kSoftcap && __all_sync(0xffffffffu, m_run != -INFINITY);
+      if (have_max) {
+        pass(-m_run, true);
+      } else {
+#pragma unroll
+        for (int c = 0; c < BN; c += 16)
+#pragma unroll
+          for (int k = 0; k < 8; ++k) mxa[k] = fmax3(mxa[k], s[c + k], s[c + 8 + k]);
+      }
+      const float mx = row_max();
+      const float mxs = mx * sc;
+      const bool move = mx > -INFINITY && (m_run == -INFINITY || mxs > m_run + kRescaleThreshold);
+      float alpha = 1.f;
+      if (__any_sync(0xffffffffu, move || !have_max)) {
+        bool rescale = false;
+        if (move) {
+          if (m_run != -INFINITY) { alpha = ex2_approx(m_run - mxs); rescale = true; }
+          m_run = mxs;
+        }
+        pass(m_run == -INFINITY ? 0.f : -m_run, false);
+        if (__any_sync(0xffffffffu, rescale)) {
+          // PV_x(j-1) is complete: this step's S-full barrier was committed after it.
+#pragma unroll 1
+          for (int q = 0; q < 4; ++q) {
+            uint32_t v[32];
+            tmem_ld32(t_o + q * 32, v);
+            tmem_ld_wait();
+#pragma unroll
+            for (int e = 0; e < 32; ++e) v[e] = __float_as_uint(__uint_as_float(v[e]) * alpha);
+            tmem_st32(t_o + q * 32, v);
+          }
         }
       }
       tmem_st_wait();

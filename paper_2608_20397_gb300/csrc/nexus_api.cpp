@@ -9,6 +9,7 @@
 
 #include <algorithm>
 #include <cmath>
+#include <cstdio>
 #include <cstring>
 #include <memory>
 #include <mutex>
@@ -740,19 +741,60 @@ nexus_status nexus_slb_quantize(const float* h_x, int32_t n, int32_t dim, int8_t
 }
 
 // Page-locked staging memory: fresh anonymous pages registered with the driver.
-static size_t host_mapping_len(size_t bytes) {
+// Mappings of at least a quarter of the transparent huge page size are rounded
+// up to whole huge pages, aligned to them and advised to use them: DMA from
+// scattered small pages ran at a few GB/s on Grace hosts, from huge pages at
+// the link rate.
+static size_t host_base_page() {
   const long pg = sysconf(_SC_PAGESIZE);
-  const size_t page = pg > 0 ? static_cast<size_t>(pg) : 4096;
-  return (bytes + page - 1) / page * page;
+  return pg > 0 ? static_cast<size_t>(pg) : 4096;
+}
+
+static size_t host_huge_page() {
+  static const size_t hp = [] {
+    size_t v = 0;
+    if (FILE* f = std::fopen("/sys/kernel/mm/transparent_hugepage/hpage_pmd_size", "r")) {
+      unsigned long long x = 0;
+      if (std::fscanf(f, "%llu", &x) == 1) v = static_cast<size_t>(x);
+      std::fclose(f);
+    }
+    const size_t base = host_base_page();
+    return (v >= base && (v & (v - 1)) == 0) ? v : 0;
+  }();
+  return hp;
+}
+
+static size_t host_mapping_len(size_t bytes, size_t* align) {
+  const size_t hp = host_huge_page();
+  const size_t unit = (hp && bytes >= hp / 4) ? hp : host_base_page();
+  *align = unit;
+  return (bytes + unit - 1) / unit * unit;
 }
 
 nexus_status nexus_host_alloc(size_t bytes, void** out) {
   if (!out) return NEXUS_EINVAL;
   *out = nullptr;
   if (bytes == 0 || bytes > (static_cast<size_t>(1) << 48)) return NEXUS_EINVAL;
-  const size_t len = host_mapping_len(bytes);
-  void* p = mmap(nullptr, len, PROT_READ | PROT_WRITE, MAP_PRIVATE | MAP_ANONYMOUS, -1, 0);
-  if (p == MAP_FAILED) return NEXUS_ENOMEM;
+  size_t align = 0;
+  const size_t len = host_mapping_len(bytes, &align);
+  const size_t extra = align > host_base_page() ? align : 0;
+  void* raw = mmap(nullptr, len + extra, PROT_READ | PROT_WRITE, MAP_PRIVATE | MAP_ANONYMOUS, -1, 0);
+  if (raw == MAP_FAILED) return NEXUS_ENOMEM;
+  uint8_t* p = static_cast<uint8_t*>(raw);
+  if (extra) {
+    // keep the aligned [p, p + len) and return the rest
+    const uintptr_t a = reinterpret_cast<uintptr_t>(raw);
+    p = reinterpret_cast<uint8_t*>((a + align - 1) / align * align);
+    const size_t head = static_cast<size_t>(p - static_cast<uint8_t*>(raw));
+    if (head) munmap(raw, head);
+    if (extra - head) munmap(p + len, extra - head);
+#ifdef MADV_HUGEPAGE
+    madvise(p, len, MADV_HUGEPAGE);   // advice only; small pages if the kernel declines
+#endif
+  }
+  // Fault every page in (zero-filled) before the driver pins them.
+  const size_t base = host_base_page();
+  for (size_t off = 0; off < len; off += base) static_cast<volatile uint8_t*>(p)[off] = 0;
   if (cudaHostRegister(p, len, cudaHostRegisterDefault) != cudaSuccess) {
     cudaGetLastError();
     munmap(p, len);
@@ -765,9 +807,11 @@ nexus_status nexus_host_alloc(size_t bytes, void** out) {
 nexus_status nexus_host_free(void* p, size_t bytes) {
   if (!p) return NEXUS_OK;
   if (bytes == 0) return NEXUS_EINVAL;
+  size_t align = 0;
+  const size_t len = host_mapping_len(bytes, &align);
   const bool unregistered = cudaHostUnregister(p) == cudaSuccess;
   if (!unregistered) cudaGetLastError();
-  munmap(p, host_mapping_len(bytes));
+  munmap(p, len);
   return unregistered ? NEXUS_OK : NEXUS_ECUDA;
 }
 

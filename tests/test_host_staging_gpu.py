@@ -52,3 +52,16 @@ def test_views_keep_the_mapping(dev):
     d = v.to(dev, non_blocking=True)
     torch.cuda.synchronize()
     assert torch.equal(d.cpu(), torch.full((10, 128), 2.5))
+
+
+def test_large_staging_region(dev):
+    # 600 MB: rounded up to whole transparent huge pages where the host has them
+    shape = (300, 1 << 20)
+    h = nexus.host_empty(shape, torch.bfloat16)
+    assert not h[::37].view(torch.int16).any()
+    d = torch.randn(shape, device=dev).to(torch.bfloat16)
+    h.copy_(d, non_blocking=True)
+    back = torch.empty_like(d)
+    back.copy_(h, non_blocking=True)
+    torch.cuda.synchronize()
+    assert torch.equal(back.view(torch.int16), d.view(torch.int16))
