@@ -434,16 +434,19 @@ attention_kernel(const __grid_constant__ AttnLaunch p, const __grid_constant__ A
     const uint64_t dv1 = vt ? smem_desc(sbase + OFF_V + kTileBytes, 16, 256, kSwizzle32B)
                             : smem_desc(sbase + OFF_V + kTileBytes, kHalf, 1024, kSwizzle128B);
     const uint64_t v_step = vt ? (4096 >> 4) : (2048 >> 4);
-    // Lanes 0-3 wait on different barriers at once (0 = none).
+    // The whole warp waits on up to four barriers with one try-wait per lane:
+    // lane l polls barrier l % 4, and a lane without one (0 = none) polls the Q
+    // barrier, complete by then. In the usual case, every barrier already
+    // complete, that is one instruction and one vote.
     auto wait4 = [&](uint32_t b0, uint32_t p0, uint32_t b1, uint32_t p1, uint32_t b2, uint32_t p2,
                      uint32_t b3, uint32_t p3) -> bool {
-      uint32_t br = 0, par = 0;
-      if (lane == 0) { br = b0; par = p0; }
-      if (lane == 1) { br = b1; par = p1; }
-      if (lane == 2) { br = b2; par = p2; }
-      if (lane == 3) { br = b3; par = p3; }
-      const bool wt = br ? mbar_wait(br, par, kBudgetNs, abort, gabort) : true;
-      __syncwarp();
+      const int l4 = lane & 3;
+      uint32_t br = l4 == 0 ? b0 : l4 == 1 ? b1 : l4 == 2 ? b2 : b3;
+      uint32_t par = l4 == 0 ? p0 : l4 == 1 ? p1 : l4 == 2 ? p2 : p3;
+      if (br == 0) { br = bar(B_Q); par = 0; }
+      bool done = mbar_try_wait(br, par);
+      if (__all_sync(0xffffffffu, done)) return true;
+      const bool wt = done || mbar_wait(br, par, kBudgetNs, abort, gabort);
       return __all_sync(0xffffffffu, wt);
     };
     bool ok = true;
