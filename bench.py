@@ -845,10 +845,10 @@ def _slb_measure(wl, stream, peaks, peak_kind, with_oracle, reps=200):
            "large": {"tools": n_big, "dim": dim, "by_batch": by_batch,
                      "note": "8 and 32 queries per launch are bound by the dp4a and shared-"
                              "memory issue rate, not by HBM"},
-           "roofline": {"bound": "hbm", "kernel": "slb_small_kernel (1M x 768 codes, 1 query)",
+           "roofline": {"bound": "hbm", "kernel": "slb_stream_kernel (1M x 768 codes, 1 query)",
                         "achieved": gbs, "peak": peaks["hbm_gbs"], "unit": "GB/s",
                         "frac": gbs / peaks["hbm_gbs"], "peak_kind": f"copy, {peak_kind}",
-                        "traffic": _profiled_traffic("slb_small_kernel")}}
+                        "traffic": _profiled_traffic("slb_stream_kernel")}}
     del big, ws_big
     if with_oracle:
         import oracle

@@ -172,9 +172,16 @@ struct SlbLaunch {
   int32_t n_queries;            // 1..32
   int32_t tools_per_cta;
   float tau;
+  int32_t chunk_tools;          // streamed scan: tools per shared-memory stage (0: not streamed)
+  int32_t stages;               // streamed scan: stages in the ring
 };
 constexpr int kSlbMaxQueries = 32;
 constexpr int kSlbSmallQueries = 4;   // up to this many queries: the latency path
+// Few queries over at least this many tools: the registry streams through
+// shared memory by bulk copies (two CTAs per SM).
+constexpr int kSlbStreamMinTools = 16384;
+constexpr int kSlbStreamSmemPerCta = 110 * 1024;  // stage ring + queries, two CTAs per SM
 cudaError_t launch_slb(const SlbLaunch& p, int grid, cudaStream_t stream);
+cudaError_t slb_take_timeout(unsigned int* flag, cudaStream_t stream);
 
 }  // namespace nexus

@@ -433,13 +433,14 @@ nexus_status attention_impl(const nexus_kv_cache* c, const int32_t* d_pt, int32_
 extern "C" {
 
 nexus_status nexus_device_status(nexus_stream stream) {
-  unsigned int flag = 0, qkv_timeout = 0, bad_page = 0;
+  unsigned int flag = 0, qkv_timeout = 0, bad_page = 0, slb_timeout = 0;
   if (attention_take_timeout(&flag, static_cast<cudaStream_t>(stream)) != cudaSuccess ||
-      qkv_take_status(&qkv_timeout, &bad_page, static_cast<cudaStream_t>(stream)) != cudaSuccess) {
+      qkv_take_status(&qkv_timeout, &bad_page, static_cast<cudaStream_t>(stream)) != cudaSuccess ||
+      slb_take_timeout(&slb_timeout, static_cast<cudaStream_t>(stream)) != cudaSuccess) {
     cudaGetLastError();
     return NEXUS_ECUDA;
   }
-  if (flag || qkv_timeout) return NEXUS_ETIMEOUT;
+  if (flag || qkv_timeout || slb_timeout) return NEXUS_ETIMEOUT;
   return bad_page ? NEXUS_ERANGE : NEXUS_OK;
 }
 
@@ -702,7 +703,28 @@ nexus_status nexus_slb_route(const int8_t* d_tools, const float* d_tool_scales, 
   for (int32_t q0 = 0; q0 < n_queries; q0 += kSlbMaxQueries) {
     p.n_queries = std::min(kSlbMaxQueries, n_queries - q0);
     int32_t per = 0;
-    const int grid = slb_grid(n_tools, p.n_queries, &per);
+    int grid = slb_grid(n_tools, p.n_queries, &per);
+    p.chunk_tools = 0;
+    p.stages = 0;
+    if (p.n_queries <= kSlbSmallQueries && n_tools >= kSlbStreamMinTools &&
+        aligned16(d_tool_scales)) {
+      // Streamed scan: stages of 8 m tools, m the largest power of two (at most
+      // 32) with about 8 KiB of codes per warp and stage, halved until two
+      // stages and the queries fit a CTA's share of the SM's shared memory
+      // (two CTAs per SM); as many stages as fit; contiguous ranges per CTA
+      // that are whole stages but the last.
+      const int kq = p.n_queries == 1 ? 1 : kSlbSmallQueries;
+      const int budget = kSlbStreamSmemPerCta - kq * dim;
+      int m = 1;
+      while (m < 32 && 2 * m * dim <= 8192) m *= 2;
+      while (m > 1 && 2 * 8 * m * (dim + 4) > budget) m /= 2;
+      const int T = 8 * m;
+      p.chunk_tools = T;
+      p.stages = std::min(8, std::max(2, budget / (T * (dim + 4))));
+      const int64_t g = std::min<int64_t>((n_tools + T - 1) / T, 2 * num_sms());
+      per = static_cast<int32_t>(((n_tools + g - 1) / g + T - 1) / T * T);
+      grid = (n_tools + per - 1) / per;
+    }
     p.tools_per_cta = per;
     p.queries = d_queries + static_cast<int64_t>(q0) * dim;
     p.query_scales = d_query_scales + q0;

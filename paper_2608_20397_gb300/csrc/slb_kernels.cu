@@ -11,7 +11,8 @@
 // integer dot of query q, so lane q keeps query q's running top two. Up to 4
 // queries (slb_small_kernel, the routing of single requests) read the query
 // words straight into registers, load all of a tool's words at once and run
-// with one or two tools per warp, for latency. Warps merge in shared memory,
+// with one or two tools per warp, for latency; over large registries they
+// stream through shared memory instead (slb_stream_kernel, below). Warps merge in shared memory,
 // CTAs write their top two per query to the workspace, and the CTA that
 // finishes last (an atomic ticket; nothing waits) merges them, applies the gate
 // and resets the ticket for the next call. The merge uses a total order (score,
@@ -19,9 +20,14 @@
 #include <cstdint>
 
 #include "internal.h"
+#include "ptx.cuh"
 
 namespace nexus {
+
+__device__ unsigned int g_slb_timeout = 0;
+
 namespace {
+using namespace ptx;
 
 constexpr int kSlbThreads = 256;
 constexpr int kSlbWarps = kSlbThreads / 32;
@@ -273,6 +279,239 @@ __global__ void __launch_bounds__(kSlbThreads) slb_small_kernel(const __grid_con
   if (s_last) final_merge(p, warp, lane);
 }
 
+// A large registry with few queries is a pure stream of HBM reads (each code
+// byte is used once per query). Each CTA owns a contiguous range of tools and
+// streams it through a ring of shared-memory stages: one thread issues a bulk
+// copy per stage as soon as the stage is free, so the copies run ahead of the
+// products without holding registers; eight warps split the stage's tools,
+// groups of lanes per tool striding over its 4-byte words, dp4a against the
+// query words held in shared memory, and a butterfly sum within the group. The stage also
+// carries the tools' scales (the scale array must be 16-byte aligned). A CTA's last,
+// partial stage is read straight from global memory (its size need not be a
+// multiple of 16 bytes). Waits are bounded; on expiry the CTA records a
+// timeout, lets its copies land and finishes the merge with what it has.
+constexpr int kStreamWarps = 8;                          // product warps
+constexpr int kStreamThreads = (kStreamWarps + 1) * 32;  // + the copy warp
+constexpr uint64_t kSlbBudgetNs = 2000000000ull;
+constexpr uint64_t kSlbDrainNs = 200000000ull;
+
+template <int kQ>
+__global__ void __launch_bounds__(kStreamThreads, 2) slb_stream_kernel(const __grid_constant__ SlbLaunch p) {
+  extern __shared__ uint8_t s_dyn[];
+  __shared__ Top2 s_top[kStreamWarps][kQ];
+  __shared__ bool s_last;
+  __shared__ int s_abort;
+  __shared__ int s_never;
+  uint8_t* s_base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(s_dyn) + 127) &
+                                               ~static_cast<uintptr_t>(127));
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  const int words = p.dim / 4;
+  const int nq = p.n_queries;
+  const int T = p.chunk_tools;
+  const int S = p.stages;
+  const uint32_t chunk_bytes = static_cast<uint32_t>(T) * p.dim;
+  const uint32_t scale_bytes = static_cast<uint32_t>(T) * 4u;
+  uint8_t* s_tools = s_base;                                                       // [S][T][dim]
+  float* s_scale = reinterpret_cast<float*>(s_base + (size_t)S * chunk_bytes);     // [S][T]
+  int32_t* s_q = reinterpret_cast<int32_t*>(s_base + (size_t)S * (chunk_bytes + scale_bytes));
+  const uint32_t bar0 = smem_u32(reinterpret_cast<uint8_t*>(s_q) + ((kQ * p.dim + 15) & ~15));
+  auto full = [&](int s) -> uint32_t { return bar0 + 8u * s; };
+  auto empty = [&](int s) -> uint32_t { return bar0 + 8u * (S + s); };
+  const volatile unsigned int* gabort = &g_slb_timeout;
+
+  const int t0 = blockIdx.x * p.tools_per_cta;
+  const int t1 = min(p.n_tools, t0 + p.tools_per_cta);
+  const int n_own = max(0, t1 - t0);
+  const int n_full = n_own / T;                 // stages copied into shared memory
+  const int n_chunks = (n_own + T - 1) / T;
+
+  const int32_t* qsrc = reinterpret_cast<const int32_t*>(p.queries);
+  for (int i = threadIdx.x; i < kQ * words; i += kStreamThreads)
+    s_q[i] = i < nq * words ? qsrc[i] : 0;
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < S; ++s) {
+      mbar_init(full(s), 1);
+      mbar_init(empty(s), kStreamWarps);
+    }
+    s_abort = 0;
+    s_never = 0;
+    fence_mbar_init();
+  }
+  __syncthreads();
+  volatile int* abort = &s_abort;
+
+  Top2 top[kQ];
+  float qscale[kQ];
+#pragma unroll
+  for (int q = 0; q < kQ; ++q) {
+    top[q] = empty_top2();
+    qscale[q] = q < nq ? __ldg(p.query_scales + q) : 0.f;
+  }
+
+  if (warp == kStreamWarps) {
+    // ---- copy warp: one thread fills the ring
+    if (lane == 0) {
+      int issued = 0;
+      for (int c = 0; c < n_full; ++c) {
+        const int s = c % S;
+        if (c >= S && !mbar_wait(empty(s), ((c / S) - 1) & 1, kSlbBudgetNs, abort, gabort)) {
+          *abort = 1;
+          atomicOr(&g_slb_timeout, 1u);
+          break;
+        }
+        mbar_arrive_expect_tx(full(s), chunk_bytes + scale_bytes);
+        bulk_load(smem_u32(s_tools + (size_t)s * chunk_bytes), p.tools + (int64_t)(t0 + c * T) * p.dim,
+                  chunk_bytes, full(s));
+        bulk_load(smem_u32(s_scale + (size_t)s * T), p.tool_scales + t0 + c * T, scale_bytes, full(s));
+        issued = c + 1;
+      }
+      // The copies issued here land before the CTA can exit.
+      for (int c = max(0, issued - S); c < issued; ++c)
+        mbar_wait(full(c % S), (c / S) & 1, kSlbDrainNs, &s_never);
+    }
+  } else {
+    // ---- product warps: warp w takes tools [w m, w m + m) of every stage,
+    // L = 32 / m lanes per tool striding over its words; each lane keeps the
+    // top two of the tools its lane group saw, merged across lanes at the end.
+    const int m = T / kStreamWarps;            // a power of two, 1..32
+    const int L = 32 / m;
+    const bool vec = (p.dim & 15) == 0;        // rows and queries in 16-byte words
+    const int n4 = p.dim / 16;
+    const int sub = lane % L;
+    const int x = warp * m + lane / L;         // this lane group's tool within a stage
+    for (int c = 0; c < n_chunks; ++c) {
+      const bool staged = c < n_full;
+      const int s = c % S;
+      if (staged) {
+        const bool ok = __all_sync(0xffffffffu, mbar_wait(full(s), (c / S) & 1, kSlbBudgetNs, abort,
+                                                          gabort));
+        if (!ok) {
+          if (lane == 0) {
+            *abort = 1;
+            atomicOr(&g_slb_timeout, 1u);
+          }
+          break;
+        }
+      }
+      const bool valid = x < min(T, n_own - c * T);
+      int acc[kQ];
+#pragma unroll
+      for (int q = 0; q < kQ; ++q) acc[q] = 0;
+      if (valid) {
+        if (staged && vec) {
+          // 16-byte words of the row and the queries, four independent chains
+          const int4* row = reinterpret_cast<const int4*>(s_tools + (size_t)s * chunk_bytes +
+                                                          (size_t)x * p.dim);
+          const int4* q4 = reinterpret_cast<const int4*>(s_q);
+          int a1[kQ], a2[kQ], a3[kQ];
+#pragma unroll
+          for (int q = 0; q < kQ; ++q) a1[q] = a2[q] = a3[q] = 0;
+#pragma unroll 2
+          for (int v = sub; v < n4; v += L) {
+            const int4 t = row[v];
+#pragma unroll
+            for (int q = 0; q < kQ; ++q) {
+              const int4 u = q4[q * n4 + v];
+              acc[q] = __dp4a(t.x, u.x, acc[q]);
+              a1[q] = __dp4a(t.y, u.y, a1[q]);
+              a2[q] = __dp4a(t.z, u.z, a2[q]);
+              a3[q] = __dp4a(t.w, u.w, a3[q]);
+            }
+          }
+#pragma unroll
+          for (int q = 0; q < kQ; ++q) acc[q] += (a1[q] + a2[q]) + a3[q];
+        } else if (staged) {
+          const int32_t* row =
+              reinterpret_cast<const int32_t*>(s_tools + (size_t)s * chunk_bytes + (size_t)x * p.dim);
+#pragma unroll 4
+          for (int w = sub; w < words; w += L) {
+            const int32_t tw = row[w];
+#pragma unroll
+            for (int q = 0; q < kQ; ++q) acc[q] = __dp4a(tw, s_q[q * words + w], acc[q]);
+          }
+        } else {
+          const int32_t* row =
+              reinterpret_cast<const int32_t*>(p.tools + ((int64_t)(t0 + c * T) + x) * p.dim);
+#pragma unroll 4
+          for (int w = sub; w < words; w += L) {
+            const int32_t tw = __ldg(row + w);
+#pragma unroll
+            for (int q = 0; q < kQ; ++q) acc[q] = __dp4a(tw, s_q[q * words + w], acc[q]);
+          }
+        }
+      }
+      const int tool = t0 + c * T + x;
+      const float ts = !valid ? 0.f : staged ? s_scale[s * T + x] : __ldg(p.tool_scales + tool);
+#pragma unroll
+      for (int q = 0; q < kQ; ++q) {
+        for (int off = L >> 1; off >= 1; off >>= 1) acc[q] += __shfl_xor_sync(0xffffffffu, acc[q], off);
+        if (valid && q < nq) push(top[q], __int2float_rn(acc[q]) * (qscale[q] * ts), tool);
+      }
+      if (staged) {
+        __syncwarp();
+        if (lane == 0) mbar_arrive(empty(s));
+      }
+    }
+    // The lanes of a group hold the same top two: one lane per group enters
+    // the merge, so every tool is counted once.
+#pragma unroll
+    for (int q = 0; q < kQ; ++q) {
+      if (sub != 0) top[q] = empty_top2();
+#pragma unroll
+      for (int off = 16; off >= 1; off >>= 1) {
+        const Top2 o = shfl_top2(top[q], off);
+        push(top[q], o.s1, o.i1);
+        push(top[q], o.s2, o.i2);
+      }
+    }
+    if (lane == 0) {
+#pragma unroll
+      for (int q = 0; q < kQ; ++q) s_top[warp][q] = top[q];
+    }
+  }
+  __syncthreads();
+  if (warp == 0) {
+    if (lane < nq) {
+      Top2 m = s_top[0][lane];
+      for (int w = 1; w < kStreamWarps; ++w) {
+        const Top2 o = s_top[w][lane];
+        push(m, o.s1, o.i1);
+        push(m, o.s2, o.i2);
+      }
+      const int64_t k = (int64_t)blockIdx.x * 32 + lane;
+      p.part_score[2 * k] = m.s1;
+      p.part_score[2 * k + 1] = m.s2;
+      p.part_idx[2 * k] = m.i1;
+      p.part_idx[2 * k + 1] = m.i2;
+    }
+    __threadfence();
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) s_last = atomicAdd(p.counter, 1u) == gridDim.x - 1;
+  __syncthreads();
+  if (s_last) final_merge(p, warp, lane);
+}
+
+size_t stream_smem_bytes(const SlbLaunch& p, int kq) {
+  return (size_t)p.stages * p.chunk_tools * (p.dim + 4) + ((kq * p.dim + 15) & ~15) +
+         16u * p.stages + 128;
+}
+
+template <int kQ>
+cudaError_t launch_stream_as(const SlbLaunch& p, int grid, cudaStream_t stream) {
+  const size_t smem = stream_smem_bytes(p, kQ);
+  cudaError_t e = cudaFuncSetAttribute(slb_stream_kernel<kQ>,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e != cudaSuccess) return e;
+  // all of the SM's unified L1 / shared storage as shared memory: two CTAs per SM
+  e = cudaFuncSetAttribute(slb_stream_kernel<kQ>, cudaFuncAttributePreferredSharedMemoryCarveout,
+                           (int)cudaSharedmemCarveoutMaxShared);
+  if (e != cudaSuccess) return e;
+  slb_stream_kernel<kQ><<<(unsigned)grid, kStreamThreads, smem, stream>>>(p);
+  return cudaGetLastError();
+}
+
 template <int kQ>
 cudaError_t launch_slb_as(const SlbLaunch& p, int grid, cudaStream_t stream) {
   const size_t smem = (size_t)kQ * p.dim;
@@ -289,6 +528,10 @@ cudaError_t launch_slb_as(const SlbLaunch& p, int grid, cudaStream_t stream) {
 
 cudaError_t launch_slb(const SlbLaunch& p, int grid, cudaStream_t stream) {
   if (p.n_queries <= 0 || grid <= 0) return cudaSuccess;
+  if (p.chunk_tools > 0) {
+    if (p.n_queries == 1) return launch_stream_as<1>(p, grid, stream);
+    return launch_stream_as<kSlbSmallQueries>(p, grid, stream);
+  }
   if (p.n_queries <= kSlbSmallQueries) {
     // Many tools per warp: four per step for more loads in flight; otherwise one
     // per warp, so a small registry spreads over every warp.
@@ -305,6 +548,14 @@ cudaError_t launch_slb(const SlbLaunch& p, int grid, cudaStream_t stream) {
   if (p.n_queries <= 8) return launch_slb_as<8>(p, grid, stream);
   if (p.n_queries <= 16) return launch_slb_as<16>(p, grid, stream);
   return launch_slb_as<32>(p, grid, stream);
+}
+
+cudaError_t slb_take_timeout(unsigned int* flag, cudaStream_t stream) {
+  cudaError_t e = cudaStreamSynchronize(stream);
+  if (e != cudaSuccess) return e;
+  if ((e = cudaMemcpyFromSymbol(flag, g_slb_timeout, sizeof(unsigned int))) != cudaSuccess) return e;
+  const unsigned int zero = 0;
+  return cudaMemcpyToSymbol(g_slb_timeout, &zero, sizeof(unsigned int));
 }
 
 }  // namespace nexus

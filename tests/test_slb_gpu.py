@@ -136,3 +136,36 @@ def test_slb_bench_size_one_million_tools(dev):
             assert (top_idx[a, 0], top_idx[a, 1]) == (i1, i2), (nq, a)
             assert top_score[a, 0] == s1 and top_score[a, 1] == s2
             assert route[a] == (i1 if np.float32(s1 - s2) > np.float32(TAU) else -1)
+
+
+@pytest.mark.parametrize("dim,n_tools", [(768, 16384 + 37), (4096, 16384 + 5), (64, 20000 + 3),
+                                         (4, 16384), (72, 40001), (768, 100_003)])
+@pytest.mark.parametrize("nq", [1, 2, 4])
+def test_slb_streamed_registry(dev, dim, n_tools, nq):
+    # Registries of 16384 tools and more with up to four queries stream through
+    # shared memory by bulk copies; each CTA's last stage may be partial and is
+    # read from global memory. Exact parity with the oracle.
+    r = np.random.default_rng(dim * 7 + n_tools + nq)
+    tc = r.integers(-127, 128, (n_tools, dim), dtype=np.int8)
+    ts = (r.random(n_tools, dtype=np.float32) * np.float32(0.01)).astype(np.float32)
+    qc = r.integers(-127, 128, (nq, dim), dtype=np.int8)
+    qs = (r.random(nq, dtype=np.float32) * np.float32(0.01)).astype(np.float32)
+    tc[n_tools - 1] = tc[3]            # a tie between the first and the last stage
+    ts[n_tools - 1] = ts[3]
+    got = run(dev, tc, ts, qc, qs)
+    assert nexus.device_status() == nexus.OK
+    check(got, tc, ts, qc, qs)
+
+
+def test_slb_streamed_workspace_reuse(dev):
+    x = tool_registry(50_000, seed=12)
+    q, _ = tool_queries(x, 3, seed=13)
+    tc, ts = oracle.slb_quantize(x)
+    qc, qs = oracle.slb_quantize(q)
+    ws = torch.zeros(nexus.slb_workspace_size(tc.shape[0]), dtype=torch.uint8, device=dev)
+    first = run(dev, tc, ts, qc, qs, ws=ws)
+    check(first, tc, ts, qc, qs)
+    second = run(dev, tc, ts, qc, qs, ws=ws)
+    for a, b in zip(first, second):
+        assert np.array_equal(a, b)
+    assert not ws[:16].any()
