@@ -398,6 +398,16 @@ def main():
                        "frac_of_8tbs_spec": splice_gbs / 8000.0,
                        "traffic": _profiled_traffic("splice_kernel")}
     suf_tflops = wl.flops_suf / (suf_ms * 1e-3) / 1e12
+    # The split-KV suffix sits near the ridge (about 320 flop per byte of K/V):
+    # both fractions, per layer. Bytes: every key's K and V row of the layer
+    # (8 KV heads x 128 x bf16, twice) plus Q read and O written.
+    suf_bytes = wl.L * (wl.T * HKV * D * 2 * 2 + 2 * wl.R_split * HQ * D * 2)
+    suf_gbs = suf_bytes / (suf_ms * 1e-3) / 1e9
+    roofline_suffix = {"kernel": "attention_kernel + combine_kernel (split-KV suffix, "
+                                 f"{wl.R_split} queries over {wl.T} keys, {wl.splits} splits)",
+                       "achieved_tflops": suf_tflops, "frac_tensor": suf_tflops / peak_tc,
+                       "achieved_gbs": suf_gbs, "frac_hbm": suf_gbs / peaks["hbm_gbs"],
+                       "peak_kind": f"bf16 sustained / copy, {peak_kind}"}
 
     e2e = None
     if not args.no_e2e:
@@ -440,7 +450,7 @@ def main():
                                 world),
             "suffix_splits": wl.splits,
             "splice_gbs": splice_gbs, "splice_ms": splice_ms, "reprefill_ms": pre_ms,
-            "suffix_ms": suf_ms, "suffix_tflops": suf_tflops,
+            "suffix_ms": suf_ms, "suffix_tflops": suf_tflops, "roofline_suffix": roofline_suffix,
             "roofline": roofline, "roofline_splice": roofline_splice,
             "e2e": e2e, "cpu_baseline": cpu, "clocks": clocks, "qkv_recompute": qkv, "l0_arena": arena, "slb_route": slb,
             "gpu_launches": wl.launches_per_step * args.steps,

@@ -151,28 +151,6 @@ __device__ __forceinline__ float fmax3(float a, float b, float c) {
   return d;
 }
 
-// 2^x on the FMA pipe, to take part of the exponentials off the MUFU unit:
-// 2^x = 2^n * 2^f with n = rint(x) (by the 1.5 * 2^23 rounding constant) and
-// f = x - n in [-0.5, 0.5]; 2^f is a degree-3 polynomial fitted here for the
-// least maximum relative error on that interval (7.5e-5, far below the bf16
-// resolution of P); n is added into the exponent field. Below 2^-125 the
-// result is exactly 0, so masked scores (-inf) still give p = 0.
-constexpr float kExp2C0 = 0.99992806f;
-constexpr float kExp2C1 = 0.69326097f;
-constexpr float kExp2C2 = 0.24261113f;
-constexpr float kExp2C3 = 0.05517167f;
-constexpr int kPolyPairsPer8 = 0;   // pairs (of every 8) whose exponentials use the polynomial
-
-__device__ __forceinline__ float exp2_poly(float x) {
-  const float xc = fmaxf(x, -125.f);
-  const float t = __fadd_rn(xc, 12582912.f);
-  const float n = __fsub_rn(t, 12582912.f);
-  const float f = __fsub_rn(xc, n);
-  const float p = fmaf(fmaf(fmaf(kExp2C3, f, kExp2C2), f, kExp2C1), f, kExp2C0);
-  const float y = __int_as_float(__float_as_int(p) + (__float_as_int(t) << 23));
-  return x < -125.f ? 0.f : y;
-}
-
 // D[tmem] (+)= A[tmem] * B[smem]: A is read from tensor memory (P, packed
 // bf16 pairs along K, row i in lane i).
 __device__ __forceinline__ void mma_bf16_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t b_desc,
