@@ -135,19 +135,20 @@ struct QkvLaunch {
   int32_t rope_gptj;
   int32_t n_tok;            // packed tokens (sum of q_len)
   int32_t k_blocks;         // ceil(hidden / 64)
-  int32_t n_tiles;          // 256-feature tiles: ceil(n_heads / 2)
+  int32_t n_tiles;          // feature tiles: ceil(n_heads / 2), or n_heads with short tiles
   int32_t m_tiles;          // 128-token tiles: ceil(n_tok / 128)
   int32_t group_m;          // token tiles per raster band
   int32_t total_tiles;      // m_tiles * n_tiles
   int32_t n_seqs;
+  int32_t short_tiles;      // n_tok <= 64: one-head tiles, 64 token rows per stage
   float inv_freq_hi[kHeadDim / 2];   // theta_i / pi = hi + lo
   float inv_freq_lo[kHeadDim / 2];
   AttnSeq seq[kMaxSeqs];
 };
 
 struct QkvMaps {
-  CUtensorMap x;            // [n_tok][hidden], box 128 x 64
-  CUtensorMap w;            // [n_heads * 128][hidden], box 256 x 64
+  CUtensorMap x;            // [n_tok][hidden], box 128 x 64 (64 x 64 for short tiles)
+  CUtensorMap w;            // [n_heads * 128][hidden], box 256 x 64 (128 x 64 for short tiles)
 };
 
 cudaError_t launch_qkv(const QkvLaunch& p, const QkvMaps& maps, int grid, cudaStream_t stream);

@@ -593,7 +593,9 @@ nexus_status nexus_suffix_qkv(const nexus_kv_cache* cache, const int32_t* d_page
     n_tok += h_q_len[s];
   }
   const int32_t n_heads = n_q_heads + 2 * cache->n_kv_heads;
-  const int64_t n_tiles = (n_heads + 1) / 2;
+  // Up to 64 tokens the launch is bound by the weight read: one-head tiles.
+  const bool short_tiles = n_tok <= 64;
+  const int64_t n_tiles = short_tiles ? n_heads : (n_heads + 1) / 2;
   const int64_t total = (n_tok + 127) / 128 * n_tiles;
   if (n_tok > 0x7FFFFFFF || total > 0x7FFFFFFF) return NEXUS_ERANGE;
   if (h_page_tables) {
@@ -638,6 +640,7 @@ nexus_status nexus_suffix_qkv(const nexus_kv_cache* cache, const int32_t* d_page
   p->group_m = std::min<int32_t>(p->m_tiles, 18);
   p->total_tiles = static_cast<int32_t>(total);
   p->n_seqs = n_seqs;
+  p->short_tiles = short_tiles ? 1 : 0;
   double inv[kHeadDim / 2];
   fill_inv_freq_over_pi(cache, inv);
   for (int i = 0; i < kHeadDim / 2; ++i) {
@@ -653,9 +656,10 @@ nexus_status nexus_suffix_qkv(const nexus_kv_cache* cache, const int32_t* d_page
     off += h_q_len[s];
   }
   QkvMaps maps;
-  if (!encode_2d_sw128(&maps.x, x, static_cast<uint64_t>(hidden), static_cast<uint64_t>(n_tok), 128) ||
+  if (!encode_2d_sw128(&maps.x, x, static_cast<uint64_t>(hidden), static_cast<uint64_t>(n_tok),
+                       short_tiles ? 64 : 128) ||
       !encode_2d_sw128(&maps.w, w_qkv, static_cast<uint64_t>(hidden),
-                       static_cast<uint64_t>(n_heads) * kHeadDim, 256))
+                       static_cast<uint64_t>(n_heads) * kHeadDim, short_tiles ? 128 : 256))
     return NEXUS_ECUDA;
   const int grid = static_cast<int>(std::min<int64_t>(total, num_sms()));
   return launch_qkv(*p, maps, grid, static_cast<cudaStream_t>(stream)) == cudaSuccess ? NEXUS_OK

@@ -7,7 +7,12 @@
 // (two heads) in bands of group_m token tiles, the token tile fastest inside a
 // band: the tiles in flight at any time share a few weight tiles and the
 // band's token rows, which stay in L2, so DRAM sees each weight tile once per
-// band rather than once per wave:
+// band rather than once per wave. Up to 64 tokens (a short re-decoded suffix)
+// the launch only streams the weight: tiles are one head wide (twice the
+// CTAs), only 64 token rows are copied per box (the products' rows 64-127
+// belong to no token and are never stored), and a stage holds four boxes of
+// consecutive hidden features, so each weight row is read 512 contiguous bytes
+// at a time:
 //   warp 0     TMA producer: X and W tiles of 64 hidden features per stage,
 //              128-byte swizzle, 4-stage ring (48 KiB a stage)
 //   warp 1     tcgen05.mma issuer (one lane): 128x256x16 bf16 products into
@@ -33,24 +38,43 @@ __device__ unsigned int g_qkv_bad_page = 0;
 namespace {
 using namespace ptx;
 
-constexpr int BM = 128;   // tokens per tile
-constexpr int BN = 256;   // output features per tile (two heads)
+constexpr int BM = 128;   // token rows of a product
 constexpr int BK = 64;    // hidden features per stage
-constexpr int kStages = 4;
 constexpr int kThreads = 192;
 constexpr int kProducerWarp = 0;
 constexpr int kMmaWarp = 1;
-constexpr uint32_t kABytes = BM * BK * 2;   // 16 KiB
-constexpr uint32_t kBBytes = BN * BK * 2;   // 32 KiB
-constexpr uint32_t kStageBytes = kABytes + kBBytes;
 constexpr uint64_t kBudgetNs = 2000000000ull;   // 2 s per wait
 constexpr uint64_t kDrainNs = 200000000ull;     // 0.2 s to drain
 
-enum { B_FULL = 0, B_EMPTY = kStages, B_AFULL = 2 * kStages, B_AEMPTY = 2 * kStages + 2,
-       B_FIN = 2 * kStages + 4, kNumBars = 2 * kStages + 5 };
-constexpr uint32_t OFF_BAR = kStages * kStageBytes;
-constexpr uint32_t OFF_MISC = OFF_BAR + kNumBars * 8;
-constexpr uint32_t kSmemBytes = OFF_MISC + 16 + 1024;   // + slack for 1024-byte alignment
+// Tile shape: kBN output features (kBN / 128 heads), kXRows token rows copied
+// per stage, kStages stages. The A operand always spans BM = 128 rows of the
+// stage; with kXRows = 64 its rows 64-127 overlap the stage's W tile and
+// produce rows of the accumulator that no token owns.
+template <int kBN, int kXRows, int kStages, int kSub = 1>
+struct QkvShape {
+  static constexpr int BN = kBN;
+  static constexpr int STAGES = kStages;
+  static constexpr int SUB = kSub;   // 64-feature boxes per stage (consecutive columns)
+  static constexpr int HEADS = kBN / 128;
+  static constexpr uint32_t kABytes = kXRows * BK * 2;      // one x box
+  static constexpr uint32_t kBBytes = kBN * BK * 2;         // one W box
+  static constexpr uint32_t kSubBytes = kABytes + kBBytes;
+  static constexpr uint32_t kStageBytes = kSub * kSubBytes;
+  static constexpr int B_FULL = 0, B_EMPTY = kStages, B_AFULL = 2 * kStages,
+                       B_AEMPTY = 2 * kStages + 2, B_FIN = 2 * kStages + 4,
+                       kNumBars = 2 * kStages + 5;
+  static constexpr uint32_t OFF_BAR = kStages * kStageBytes;
+  static constexpr uint32_t OFF_MISC = OFF_BAR + kNumBars * 8;
+  static constexpr uint32_t kSmemBytes = OFF_MISC + 16 + 1024;   // + slack for 1024-byte alignment
+  static_assert(kXRows == BM || (kXRows == 64 && kSubBytes >= BM * BK * 2),
+                "the A operand's 128 rows must lie inside the sub-stage");
+  static_assert(kSubBytes % 1024 == 0 && kABytes % 1024 == 0, "128-byte swizzle atoms");
+};
+using LongTiles = QkvShape<256, 128, 4, 1>;   // 128 tokens x two heads, 4 stages of 48 KiB
+// Up to 64 tokens x one head: 2 stages of four consecutive 64-feature boxes
+// (96 KiB), so each weight row is read 512 contiguous bytes at a time (one
+// box per stage, 128 bytes per row and stage, ran 44 % slower).
+using ShortTiles = QkvShape<128, 64, 2, 4>;
 
 __device__ __forceinline__ void record_timeout(volatile int* abort) {
   *abort = 1;
@@ -90,8 +114,19 @@ __device__ __forceinline__ void tile_coords(const QkvLaunch& p, int t, int& mt, 
   nt = local / gm;
 }
 
+template <class Sh>
 __global__ void __launch_bounds__(kThreads, 1)
 qkv_kernel(const __grid_constant__ QkvLaunch p, const __grid_constant__ QkvMaps maps) {
+  constexpr int BN = Sh::BN;
+  constexpr int kStages = Sh::STAGES;
+  constexpr uint32_t kABytes = Sh::kABytes;
+  constexpr uint32_t kStageBytes = Sh::kStageBytes;
+  constexpr int kSub = Sh::SUB;
+  constexpr uint32_t kSubBytes = Sh::kSubBytes;
+  const int kb_stages = (p.k_blocks + kSub - 1) / kSub;
+  constexpr int B_FULL = Sh::B_FULL, B_EMPTY = Sh::B_EMPTY, B_AFULL = Sh::B_AFULL,
+                B_AEMPTY = Sh::B_AEMPTY, B_FIN = Sh::B_FIN;
+  constexpr uint32_t OFF_BAR = Sh::OFF_BAR, OFF_MISC = Sh::OFF_MISC;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
@@ -138,7 +173,7 @@ qkv_kernel(const __grid_constant__ QkvLaunch p, const __grid_constant__ QkvMaps 
       for (int t = blockIdx.x; t < p.total_tiles && ok; t += gridDim.x) {
         int mt, nt;
         tile_coords(p, t, mt, nt);
-        for (int kb = 0; kb < p.k_blocks; ++kb, ++it) {
+        for (int kb = 0; kb < kb_stages; ++kb, ++it) {
           const int st = it % kStages;
           if (it >= kStages) {
             ok = mbar_wait(bar(B_EMPTY + st), ((it / kStages) - 1) & 1, kBudgetNs, abort, gabort);
@@ -146,8 +181,12 @@ qkv_kernel(const __grid_constant__ QkvLaunch p, const __grid_constant__ QkvMaps 
           }
           const uint32_t a = sbase + st * kStageBytes;
           mbar_arrive_expect_tx(bar(B_FULL + st), kStageBytes);
-          tma_load_2d(a, &maps.x, bar(B_FULL + st), kb * BK, mt * BM);
-          tma_load_2d(a + kABytes, &maps.w, bar(B_FULL + st), kb * BK, nt * BN);
+#pragma unroll
+          for (int sub = 0; sub < kSub; ++sub) {
+            tma_load_2d(a + sub * kSubBytes, &maps.x, bar(B_FULL + st), (kb * kSub + sub) * BK, mt * BM);
+            tma_load_2d(a + sub * kSubBytes + kABytes, &maps.w, bar(B_FULL + st), (kb * kSub + sub) * BK,
+                        nt * BN);
+          }
         }
       }
       // The last copies issued land before the CTA can exit (at once when the
@@ -175,16 +214,19 @@ qkv_kernel(const __grid_constant__ QkvLaunch p, const __grid_constant__ QkvMaps 
         }
         tc_fence_after();
         const uint32_t d = tmem + buf * BN;
-        for (int kb = 0; kb < p.k_blocks; ++kb, ++it) {
+        for (int kb = 0; kb < kb_stages; ++kb, ++it) {
           const int st = it % kStages;
           ok = mbar_wait(bar(B_FULL + st), (it / kStages) & 1, kBudgetNs, abort, gabort);
           if (!ok) { record_timeout(abort); break; }
           tc_fence_after();
-          const uint64_t so = static_cast<uint64_t>((st * kStageBytes) >> 4);
 #pragma unroll
-          for (int kk = 0; kk < BK / 16; ++kk)
-            mma_bf16(d, da0 + so + (kk * 32 >> 4), db0 + so + (kk * 32 >> 4), idesc,
-                     (kb | kk) != 0 ? 1u : 0u);
+          for (int sub = 0; sub < kSub; ++sub) {
+            const uint64_t so = static_cast<uint64_t>((st * kStageBytes + sub * kSubBytes) >> 4);
+#pragma unroll
+            for (int kk = 0; kk < BK / 16; ++kk)
+              mma_bf16(d, da0 + so + (kk * 32 >> 4), db0 + so + (kk * 32 >> 4), idesc,
+                       (kb | sub | kk) != 0 ? 1u : 0u);
+          }
           mma_commit(bar(B_EMPTY + st));
         }
         if (ok) mma_commit(bar(B_AFULL + buf));
@@ -233,7 +275,7 @@ qkv_kernel(const __grid_constant__ QkvLaunch p, const __grid_constant__ QkvMaps 
       const int slot = pos % kPageSize;
       const float pf = static_cast<float>(pos);
       const uint32_t t_acc = tmem + lane_base + buf * BN;
-      const bool any_rot = 2 * nt < p.n_q_heads + p.n_kv_heads;
+      const bool any_rot = Sh::HEADS * nt < p.n_q_heads + p.n_kv_heads;
 
 #pragma unroll 1
       for (int c = 0; c < 2; ++c) {
@@ -254,8 +296,8 @@ qkv_kernel(const __grid_constant__ QkvLaunch p, const __grid_constant__ QkvMaps 
         const int col_a = gptj ? c * 64 : c * 32;
         const int col_b = gptj ? c * 64 + 32 : 64 + c * 32;
 #pragma unroll 1
-        for (int h = 0; h < 2; ++h) {
-          const int head = 2 * nt + h;
+        for (int h = 0; h < Sh::HEADS; ++h) {
+          const int head = Sh::HEADS * nt + h;
           if (head >= p.n_heads) break;
           __syncwarp();
           uint32_t ra[32], rb[32];
@@ -325,16 +367,22 @@ qkv_kernel(const __grid_constant__ QkvLaunch p, const __grid_constant__ QkvMaps 
   if (warp == kMmaWarp) tmem_dealloc(tmem, 512);
 }
 
+template <class Sh>
+cudaError_t launch_qkv_as(const QkvLaunch& p, const QkvMaps& maps, int grid, cudaStream_t stream) {
+  static_assert(Sh::kSmemBytes <= 227 * 1024, "shared memory budget");
+  cudaError_t e = cudaFuncSetAttribute(qkv_kernel<Sh>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       (int)Sh::kSmemBytes);
+  if (e != cudaSuccess) return e;
+  qkv_kernel<Sh><<<(unsigned)grid, kThreads, Sh::kSmemBytes, stream>>>(p, maps);
+  return cudaGetLastError();
+}
+
 }  // namespace
 
 cudaError_t launch_qkv(const QkvLaunch& p, const QkvMaps& maps, int grid, cudaStream_t stream) {
   if (p.total_tiles <= 0 || grid <= 0) return cudaSuccess;
-  static_assert(kSmemBytes <= 227 * 1024, "shared memory budget");
-  cudaError_t e = cudaFuncSetAttribute(qkv_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       (int)kSmemBytes);
-  if (e != cudaSuccess) return e;
-  qkv_kernel<<<(unsigned)grid, kThreads, kSmemBytes, stream>>>(p, maps);
-  return cudaGetLastError();
+  return p.short_tiles ? launch_qkv_as<ShortTiles>(p, maps, grid, stream)
+                       : launch_qkv_as<LongTiles>(p, maps, grid, stream);
 }
 
 cudaError_t qkv_take_status(unsigned int* timeout, unsigned int* bad_page, cudaStream_t stream) {

@@ -236,3 +236,32 @@ def test_qkv_bench_size_32768_tokens_sampled(dev):
                                              [0, 1, 127, 128, 32767, 32640]])))
     c.check(rows=rows, what="32768 tokens")
     c.check_untouched()
+
+
+@pytest.mark.parametrize("vt,gptj", [(False, False), (True, False), (True, True)])
+def test_qkv_short_suffix_64_tokens(dev, vt, gptj):
+    # 64 tokens or fewer take one-head tiles with 64 token rows per stage: the
+    # c5 suffix shape (64 re-decoded tokens, hidden 5120, 40 + 8 + 8 heads).
+    c = QkvCase(dev, [34816], [64], HIDDEN, vt=vt, gptj=gptj, seed=31, n_layers=1, layer=0)
+    c.run()
+    torch.cuda.synchronize()
+    c.check(what=f"64 tokens vt={vt} gptj={gptj}")
+    c.check_untouched()
+
+
+def test_qkv_short_suffix_ragged_sequences(dev):
+    # 63 tokens from four sequences (one empty), odd head counts, hidden 1000
+    c = QkvCase(dev, [100, 40, 5000, 17], [30, 0, 32, 1], 1000, n_q_heads=5, n_kv_heads=1,
+                vt=True, seed=32)
+    c.run()
+    torch.cuda.synchronize()
+    c.check(what="short ragged")
+    c.check_untouched()
+
+
+def test_qkv_65_tokens_take_long_tiles(dev):
+    c = QkvCase(dev, [300], [65], 512, seed=33)
+    c.run()
+    torch.cuda.synchronize()
+    c.check(what="65 tokens")
+    c.check_untouched()
