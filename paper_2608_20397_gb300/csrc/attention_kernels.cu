@@ -661,7 +661,9 @@ attention_kernel(const __grid_constant__ AttnLaunch p, const __grid_constant__ A
 
 // Merge of split-KV partials: one warp per (layer, token, head) row. Lane s
 // holds split s's LSE; the max and the weight sum are warp-shuffle
-// reductions, then every lane accumulates its four columns over the splits.
+// reductions, then every lane accumulates its four columns over the splits,
+// eight splits' loads in flight at a time (they are independent; a loop of one
+// load at a time waited out an L2 round trip per split).
 __global__ void __launch_bounds__(128) combine_kernel(const __grid_constant__ AttnLaunch p) {
   const int64_t rows = (int64_t)p.n_layers_call * p.n_tok * p.n_q_heads;
   const int64_t row = (int64_t)blockIdx.x * 4 + (threadIdx.x >> 5);
@@ -676,11 +678,23 @@ __global__ void __launch_bounds__(128) combine_kernel(const __grid_constant__ At
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) wsum += __shfl_xor_sync(0xffffffffu, wsum, o);
   float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-  for (int s = 0; s < p.splits; ++s) {
-    const float ws = __shfl_sync(0xffffffffu, w, s);
-    if (ws == 0.f) continue;
-    const float4 v = reinterpret_cast<const float4*>(p.part_o + ((int64_t)s * rows + row) * D)[lane];
-    acc.x += ws * v.x; acc.y += ws * v.y; acc.z += ws * v.z; acc.w += ws * v.w;
+  for (int s0 = 0; s0 < p.splits; s0 += 8) {
+    float4 v[8];
+    float ws[8];
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {
+      const int s = s0 + k;
+      ws[k] = __shfl_sync(0xffffffffu, w, s & 31);
+      v[k] = (s < p.splits && ws[k] != 0.f)
+                 ? __ldcg(reinterpret_cast<const float4*>(p.part_o + ((int64_t)s * rows + row) * D) + lane)
+                 : make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {
+      if (s0 + k < p.splits && ws[k] != 0.f) {
+        acc.x += ws[k] * v[k].x; acc.y += ws[k] * v[k].y; acc.z += ws[k] * v[k].z; acc.w += ws[k] * v[k].w;
+      }
+    }
   }
   const float inv = wsum > 0.f ? 1.f / wsum : 0.f;
   uint2 outv = make_uint2(pack_bf16x2(acc.x * inv, acc.y * inv), pack_bf16x2(acc.z * inv, acc.w * inv));
