@@ -160,6 +160,15 @@ int32_t nexus_version(void);
  * stream reports an error, else NEXUS_OK. */
 nexus_status nexus_device_status(nexus_stream stream);
 
+/* Self-test of the failure path above, for callers that want to see it work on
+ * their GPU: launches one CTA whose thread waits, with the same bounded
+ * mbarrier wait the kernels use, on a barrier that nothing arrives on. The wait
+ * gives up after budget_us microseconds and records a timeout, so the next
+ * nexus_device_status returns NEXUS_ETIMEOUT (and clears the record) while the
+ * context stays usable. budget_us must lie in [1, 1000000]; NEXUS_EINVAL
+ * otherwise, NEXUS_ECUDA if the launch fails. */
+nexus_status nexus_selftest_wait(uint32_t budget_us, nexus_stream stream);
+
 /* ---------------------------------------------------------------- policy */
 /* R(n_past) of Eq. 2 (Sec. III-C) as an exact fraction *num / *den in percent,
  * clamped to 100. Returns NEXUS_EINVAL for K < 2, M < 1 or R_base outside [0, 100]. */

@@ -702,7 +702,24 @@ __global__ void __launch_bounds__(128) combine_kernel(const __grid_constant__ At
   if (p.lse && lane == 0) p.lse[row] = wsum > 0.f ? mx + logf(wsum) : -INFINITY;
 }
 
+// The failure path on its own: a bounded wait on a barrier that nothing
+// arrives on gives up and records a timeout like any kernel's wait would.
+__global__ void wait_selftest_kernel(uint64_t budget_ns) {
+  __shared__ uint64_t bar_word;
+  __shared__ int abort_flag;
+  const uint32_t b = smem_u32(&bar_word);
+  mbar_init(b, 1);
+  abort_flag = 0;
+  fence_mbar_init();
+  if (!mbar_wait(b, 0, budget_ns, &abort_flag)) record_timeout(&abort_flag);
+}
+
 }  // namespace
+
+cudaError_t launch_wait_selftest(uint64_t budget_ns, cudaStream_t stream) {
+  wait_selftest_kernel<<<1, 1, 0, stream>>>(budget_ns);
+  return cudaGetLastError();
+}
 
 cudaError_t launch_attention(const AttnLaunch& p, const AttnMaps& maps, cudaStream_t stream) {
   if (p.total_tiles <= 0 || p.n_layers_call <= 0) return cudaSuccess;

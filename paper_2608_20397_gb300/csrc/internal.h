@@ -117,6 +117,8 @@ cudaError_t launch_attention(const AttnLaunch& p, const AttnMaps& maps, cudaStre
 cudaError_t launch_attn_combine(const AttnLaunch& p, cudaStream_t stream);
 // Reads and clears the timeout record of the current device.
 cudaError_t attention_take_timeout(unsigned int* flag, cudaStream_t stream);
+// One CTA waits, bounded by budget_ns, on a barrier nothing arrives on.
+cudaError_t launch_wait_selftest(uint64_t budget_ns, cudaStream_t stream);
 
 // ------------------------------------------------- suffix Q/K/V recompute
 struct QkvLaunch {

@@ -444,6 +444,14 @@ nexus_status nexus_device_status(nexus_stream stream) {
   return bad_page ? NEXUS_ERANGE : NEXUS_OK;
 }
 
+nexus_status nexus_selftest_wait(uint32_t budget_us, nexus_stream stream) {
+  if (budget_us < 1 || budget_us > 1000000) return NEXUS_EINVAL;
+  return launch_wait_selftest(static_cast<uint64_t>(budget_us) * 1000u,
+                              static_cast<cudaStream_t>(stream)) == cudaSuccess
+             ? NEXUS_OK
+             : NEXUS_ECUDA;
+}
+
 nexus_status nexus_splice_kv(const nexus_kv_cache* cache, const int32_t* d_page_tables,
                              const int32_t* h_page_tables, int32_t n_rows, int32_t max_pages,
                              const nexus_block* blocks, int32_t n_blocks,

@@ -134,6 +134,7 @@ _SIGS = {
     "nexus_suffix_qkv": (c_int32, [POINTER(KvCache), c_void_p, _i32p, c_int32, c_int32, c_int32,
                                    _i32p, _i32p, _i32p, c_void_p, c_int32, c_void_p, c_void_p,
                                    c_int32, c_int32, c_void_p, c_void_p]),
+    "nexus_selftest_wait": (c_int32, [ctypes.c_uint32, c_void_p]),
     "nexus_host_alloc": (c_int32, [c_size_t, POINTER(c_void_p)]),
     "nexus_host_free": (c_int32, [c_void_p, c_size_t]),
 }
@@ -425,6 +426,12 @@ def reprefill(cache: KvCache, d_page_tables, n_rows: int, max_pages: int, kv_len
 def device_status(stream=None) -> int:
     """Synchronises the stream; OK, ETIMEOUT (a bounded device wait gave up) or ECUDA."""
     return int(lib().nexus_device_status(_stream(stream)))
+
+
+def selftest_wait(budget_us: int = 2000, stream=None) -> None:
+    """Launches the bounded-wait self-test (see nexus_selftest_wait): the next
+    device_status() reports ETIMEOUT."""
+    _check("nexus_selftest_wait", lib().nexus_selftest_wait(int(budget_us), _stream(stream)))
 
 
 def suffix_attention_noalloc(cache: KvCache, d_page_tables, n_rows: int, max_pages: int, kv_len,

@@ -398,3 +398,9 @@ def test_host_staging_argument_checks():
         assert L.nexus_host_alloc(1 << 20, ctypes.byref(out)) == nexus.ECUDA and not out.value
         with pytest.raises(nexus.NexusError):
             nexus.host_empty((4, 4), torch.bfloat16)
+
+
+def test_selftest_wait_argument_checks():
+    L = nexus.lib()
+    assert L.nexus_selftest_wait(0, None) == nexus.EINVAL
+    assert L.nexus_selftest_wait(1000001, None) == nexus.EINVAL
