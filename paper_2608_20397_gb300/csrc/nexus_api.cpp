@@ -297,7 +297,12 @@ nexus_status plan_attention(int32_t n_seqs, const int32_t* kv_len, const int32_t
   pl.total_tiles = static_cast<int32_t>(tiles);
   if (split_kv < 0) return NEXUS_EINVAL;
   if (split_kv == 0) {
-    // Balance waves of one-CTA-per-SM work against the per-split merge.
+    // Balance waves of one-CTA-per-SM work against the per-split merge. A CTA
+    // also pays a fixed start (Q and the first K/V tiles, filling the pipeline)
+    // and end (its partial rows): about four key tiles' worth, measured on the
+    // c5 suffix (64 queries over 34816 keys: 9 splits in one wave 72 us a
+    // layer, 19 splits in two waves 84 us).
+    constexpr double kCtaFixedTiles = 4.0;
     const int64_t ctas = tiles * n_kv_heads * std::max(1, n_layers_call);
     const int sms = num_sms();
     int best = 1;
@@ -307,7 +312,8 @@ nexus_status plan_attention(int32_t n_seqs, const int32_t* kv_len, const int32_t
     if (ctas > 0 && ctas < sms && pl.kt_max > 0) {
       for (int s = 1; s <= std::min<int>(kMaxSplits, pl.kt_max); ++s) {
         const double waves = std::ceil(static_cast<double>(ctas) * s / sms);
-        const double cost = waves * std::ceil(static_cast<double>(pl.kt_max) / s) + (s > 1 ? 2.0 : 0.0);
+        const double cost = waves * (std::ceil(static_cast<double>(pl.kt_max) / s) + kCtaFixedTiles) +
+                            (s > 1 ? 2.0 : 0.0);
         if (cost < best_cost - 1e-9) { best_cost = cost; best = s; }
       }
     }
