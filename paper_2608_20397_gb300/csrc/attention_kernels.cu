@@ -519,11 +519,11 @@ attention_kernel(const __grid_constant__ AttnLaunch p, const __grid_constant__ A
         for (int c = 0; c < BN; ++c) s[c] = (c <= lim) ? s[c] : -INFINITY;
       }
       // One pass over the row: exponentials 2^(s sc - m) written to TMEM as
-      // bf16 P over the first 64 columns of S, four pair chains of the row sum,
-      // and, when `track`, the row max alongside (eight 3-input chains).
+      // bf16 P over the first 64 columns of S, and four pair chains of the row
+      // sum.
       float2 sum[4];
       float mxa[8];
-      auto pass = [&](float neg_m, bool track) {
+      auto pass = [&](float neg_m) {
         const float2 sc2 = make_float2(sc, sc);
         const float2 nm2 = make_float2(neg_m, neg_m);
 #pragma unroll
@@ -534,7 +534,6 @@ attention_kernel(const __grid_constant__ AttnLaunch p, const __grid_constant__ A
 #pragma unroll
           for (int e = 0; e < 16; e += 2) {
             const int c = q * 16 + e;
-            if (track) mxa[e >> 1] = fmax3(mxa[e >> 1], s[c], s[c + 1]);
             float2 ab = ffma2(make_float2(s[c], s[c + 1]), sc2, nm2);
             ab.x = ex2_approx(ab.x);
             ab.y = ex2_approx(ab.y);
@@ -553,15 +552,22 @@ attention_kernel(const __grid_constant__ AttnLaunch p, const __grid_constant__ A
       // The running max moves only when a tile's max exceeds it by more than
       // 2^8, which after a row's first tile is rare. So once every row of the
       // warp has a running max, the exponentials are taken with it straight
-      // away and the tile's max is tracked alongside; only if it has grown past
-      // the threshold is the pass redone with the new max. Either way the
-      // result is that of taking the max first.
-      // (Soft-capped scores always take the max first: the tracked pass holds
-      // too many registers beside the capping arithmetic.)
+      // away: if none of them exceeds 2^8 the max would not have moved, and a
+      // row sum below 2^8 proves that. A row whose sum reaches 2^8 (or is not
+      // a number) is redone with the max taken first, so the result is always
+      // that of taking the max first.
+      // (Soft-capped scores always take the max first: the speculative pass
+      // holds too many registers beside the capping arithmetic.)
       const bool have_max = !kSoftcap && __all_sync(0xffffffffu, m_run != -INFINITY);
+      bool check = true;
       if (have_max) {
-        pass(-m_run, true);
-      } else {
+        pass(-m_run);
+        const float rowsum = ((sum[0].x + sum[0].y) + (sum[1].x + sum[1].y)) +
+                             ((sum[2].x + sum[2].y) + (sum[3].x + sum[3].y));
+        check = !(rowsum < 256.f);
+      }
+      float alpha = 1.f;
+      if (__any_sync(0xffffffffu, check)) {
 #pragma unroll
         for (int c = 0; c < BN; c += 16)
 #pragma unroll
@@ -570,14 +576,13 @@ attention_kernel(const __grid_constant__ AttnLaunch p, const __grid_constant__ A
       const float mx = row_max();
       const float mxs = mx * sc;
       const bool move = mx > -INFINITY && (m_run == -INFINITY || mxs > m_run + kRescaleThreshold);
-      float alpha = 1.f;
       if (__any_sync(0xffffffffu, move || !have_max)) {
         bool rescale = false;
         if (move) {
           if (m_run != -INFINITY) { alpha = ex2_approx(m_run - mxs); rescale = true; }
           m_run = mxs;
         }
-        pass(m_run == -INFINITY ? 0.f : -m_run, false);
+        pass(m_run == -INFINITY ? 0.f : -m_run);
         if (__any_sync(0xffffffffu, rescale)) {
           // PV_x(j-1) is complete: this step's S-full barrier was committed after it.
 #pragma unroll 1
