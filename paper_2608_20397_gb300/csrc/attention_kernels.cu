@@ -496,21 +496,32 @@ attention_kernel(const __grid_constant__ AttnLaunch p, const __grid_constant__ A
           for (int e = 0; e < 32; ++e) s[q * 32 + e] = __uint_as_float(v[q][e]);
       }
       if constexpr (kSoftcap) {
-        // tanh(x) = 1 - 2 / (2^(2x log2 e) + 1) on pairs: the scaling, the +1 and
-        // the final 1 - 2r on the packed float32 pipe, ex2 and rcp on MUFU
-        const float2 ci = make_float2(p.softcap_in, p.softcap_in);
-        const float2 one = make_float2(1.f, 1.f), m2 = make_float2(-2.f, -2.f);
+        // tanh(x) = 2 / (2 z) - 1 with 2 z = 1 + u, u = 2^(-2 x log2 e); the
+        // argument is clamped at 30 so that u stays finite (and a NaN score of an
+        // unused slot, masked below, becomes a finite number). The reciprocals of a
+        // group of four z come from one: 1 / z_i = (product of the other three) /
+        // (product of all four).
+        const float2 nci = make_float2(-p.softcap_in, -p.softcap_in);
+        const float2 half = make_float2(0.5f, 0.5f), mone = make_float2(-1.f, -1.f);
 #pragma unroll
-        for (int c = 0; c < BN; c += 2) {
-          float2 e = fmul2(make_float2(s[c], s[c + 1]), ci);
-          e.x = ex2_approx(e.x);
-          e.y = ex2_approx(e.y);
-          e = fadd2(e, one);
-          e.x = rcp_approx(e.x);
-          e.y = rcp_approx(e.y);
-          e = ffma2(m2, e, one);
-          s[c] = e.x;
-          s[c + 1] = e.y;
+        for (int c = 0; c < BN; c += 4) {
+          float2 a = fmul2(make_float2(s[c], s[c + 1]), nci);
+          float2 b = fmul2(make_float2(s[c + 2], s[c + 3]), nci);
+          a.x = ex2_approx(fminf(a.x, 30.f));
+          a.y = ex2_approx(fminf(a.y, 30.f));
+          b.x = ex2_approx(fminf(b.x, 30.f));
+          b.y = ex2_approx(fminf(b.y, 30.f));
+          const float2 za = ffma2(a, half, half);
+          const float2 zb = ffma2(b, half, half);
+          const float2 zp = fmul2(za, zb);
+          const float r = rcp_approx(zp.x * zp.y);
+          const float2 rp = make_float2(r * zp.y, r * zp.x);
+          const float2 ta = fadd2(fmul2(rp, zb), mone);
+          const float2 tb = fadd2(fmul2(rp, za), mone);
+          s[c] = ta.x;
+          s[c + 1] = ta.y;
+          s[c + 2] = tb.x;
+          s[c + 3] = tb.y;
         }
       }
       const int lim = pos_r - (w.kt_begin + j) * BN;   // keys c <= lim are visible
@@ -556,9 +567,7 @@ attention_kernel(const __grid_constant__ AttnLaunch p, const __grid_constant__ A
       // row sum below 2^8 proves that. A row whose sum reaches 2^8 (or is not
       // a number) is redone with the max taken first, so the result is always
       // that of taking the max first.
-      // (Soft-capped scores always take the max first: the speculative pass
-      // holds too many registers beside the capping arithmetic.)
-      const bool have_max = !kSoftcap && __all_sync(0xffffffffu, m_run != -INFINITY);
+      const bool have_max = __all_sync(0xffffffffu, m_run != -INFINITY);
       bool check = true;
       if (have_max) {
         pass(-m_run);
