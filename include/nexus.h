@@ -364,8 +364,9 @@ nexus_status nexus_copy_pages(const nexus_kv_cache* cache, const int32_t* h_src_
  *                  back to back along the token axis in order
  *   lse            device float (nullable)
  *   n_seqs         1 .. 512
- *   split_kv       number of key-range partitions: 1 = none, 0 = chosen by
- *                  the library from the work size and SM count, up to 64
+ *   split_kv       number of key-range partitions: 1 = none, 2 .. 32 as
+ *                  given (larger values are taken as 32), 0 = chosen by the
+ *                  library from the work size and SM count (at most 32)
  *   workspace      device scratch for split partials (nullable when no split
  *                  is used); its size comes from nexus_attention_workspace_size
  *                  with the same arguments; NEXUS_ENOMEM if too small
@@ -472,7 +473,8 @@ nexus_status nexus_slb_route(const int8_t* d_tools, const float* d_tool_scales, 
 /* Bytes of workspace nexus_suffix_attention needs for these arguments
  * (0 when no split is used). *splits_out (nullable) receives the partition
  * count the call will use. Uses the current device's SM count, or 152 when no
- * device is visible. */
+ * device is visible. Arguments the attention call would reject (n_seqs outside
+ * 1 .. 512, q_len > kv_len, bad head counts) give 0 and *splits_out = 0. */
 size_t nexus_attention_workspace_size(int32_t n_seqs, const int32_t* h_kv_len,
                                       const int32_t* h_q_len, int32_t n_q_heads,
                                       int32_t n_kv_heads, int32_t n_layers_call,

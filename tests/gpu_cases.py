@@ -6,8 +6,9 @@ Tolerances (written here once, used by every GPU test):
 * re-rotated K (bf16 store): |K - K_oracle| <= 2e-3 + half a bf16 ulp of
   |K_oracle| (the bf16 store alone errs by up to half an ulp, 3.9e-3 at
   |k| in [1, 2)); the float32 output of the same arithmetic: <= 2e-3;
-* attention output: max abs <= 1e-2 and relative L2 <= 5e-3; LSE max abs
-  <= 1e-2.
+* attention output (bf16 store): |O - O_oracle| <= 1e-2 + half a bf16 ulp of
+  |O_oracle| (the store alone errs by up to half an ulp, 1.6e-2 at |o| in
+  [4, 8)) and relative L2 <= 5e-3; LSE max abs <= 1e-2.
 """
 from __future__ import annotations
 
@@ -41,7 +42,8 @@ def assert_k_close(got: np.ndarray, want: np.ndarray, what=""):
 def assert_attn_close(got: np.ndarray, want: np.ndarray, got_lse=None, want_lse=None, what=""):
     err = np.abs(got - want)
     rel = np.linalg.norm(got - want) / max(np.linalg.norm(want), 1e-30)
-    assert err.max() <= ATTN_ABS, f"{what}: max abs {err.max():.3e}"
+    bad = err > ATTN_ABS + half_ulp_bf16(want)
+    assert not bad.any(), f"{what}: {bad.sum()} outputs out of tolerance, max abs {err.max():.3e}"
     assert rel <= ATTN_REL, f"{what}: rel L2 {rel:.3e}"
     if got_lse is not None:
         e = np.abs(got_lse - want_lse)

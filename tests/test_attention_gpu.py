@@ -115,6 +115,19 @@ def test_split_kv_auto_varlen():
         _check(ks, vs, q, o, lse, kv, ql, 5, layer, what="auto split")
 
 
+def test_max_sequences_per_call():
+    """512 sequences, the most one call takes: short ragged caches, some with no
+    queries; every row against the oracle, without and with a split."""
+    rng = np.random.default_rng(21)
+    kv = [int(x) for x in rng.integers(1, 161, 512)]
+    ql = [int(rng.integers(0, min(k, 40) + 1)) for k in kv]
+    ql[0], ql[511] = 0, kv[511]
+    cache, d_pt, mp, ks, vs, q = _direct_case(kv, ql, seed=21)
+    for split in (1, 3):
+        o, lse = _run(cache, d_pt, mp, kv, ql, q, 40, 1, split_kv=split)
+        _check(ks, vs, q, o, lse, kv, ql, 5, what=f"512 sequences, split {split}")
+
+
 def test_reprefill_equals_textbook_causal():
     T = 600
     cache, d_pt, mp, ks, vs, q = _direct_case([T], [T], seed=13)

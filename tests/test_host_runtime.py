@@ -307,6 +307,19 @@ def test_workspace_size_and_split_choice():
     assert s == 1 and n == 0
     n, s = nexus.attention_workspace_size([34816], [64], 40, 8, 1, 7)
     assert s == 7 and n == 7 * 64 * 40 * 516
+    n, s = nexus.attention_workspace_size([34816], [64], 40, 8, 1, 100)   # taken as 32
+    assert s == 32 and n == 32 * 64 * 40 * 516
+    n, s = nexus.attention_workspace_size([10] * 512, [1] * 512, 40, 8, 1, 1)
+    assert s == 1 and n == 0
+    assert nexus.attention_workspace_size([10] * 513, [1] * 513, 40, 8, 1, 1) == (0, 0)
+    assert nexus.attention_workspace_size([10], [11], 40, 8, 1, 1) == (0, 0)
+
+
+def test_attention_rejects_more_than_512_sequences():
+    with pytest.raises(nexus.NexusError) as e:
+        nexus.suffix_attention(_cache(), FAKE, 513, 8, [10] * 513, [1] * 513, FAKE, FAKE,
+                               stream=0)
+    assert e.value.code == nexus.EINVAL
 
 
 def test_softcap_must_be_positive():
