@@ -902,16 +902,19 @@ def _e2e(wl, stream, args, barrier, world, dist, dev):
     nexus = wl.nexus
     # Host buffers in the library's page-locked staging memory (nexus_host_alloc,
     # huge pages where the request is large): every layer's Q in one region, the
-    # two O buffers in another.
+    # two O buffers in another, the rest in a third.
+    # The block K/V and the suffix's Q and O share one region, so that they sit in
+    # huge pages too (each alone is under the size that gets them).
     host = lambda shape, dtype=torch.bfloat16: nexus.host_empty(shape, dtype)
-    h_bk, h_bv = host(wl.bk.shape), host(wl.bv.shape)
+    bf16 = torch.bfloat16
+    h_bk, h_bv, h_qs, h_os = nexus.host_empty_group(
+        [(wl.bk.shape, bf16), (wl.bv.shape, bf16), (wl.q_suf.shape, bf16), (wl.o_suf.shape, bf16)])
     h_bk.copy_(wl.bk)
     h_bv.copy_(wl.bv)
     h_qall = host(wl.q_pre.shape)
     h_q = [h_qall[l] for l in range(L)]
     h_oall = host((2,) + tuple(wl.o_pre.shape[1:]))
     h_o = [h_oall[0], h_oall[1]]
-    h_qs, h_os = host(wl.q_suf.shape), host(wl.o_suf.shape)
     h_qall.copy_(wl.q_pre)
     h_qs.copy_(wl.q_suf)
     qbuf = [torch.empty_like(wl.q_pre[:1]) for _ in range(2)]
@@ -923,14 +926,15 @@ def _e2e(wl, stream, args, barrier, world, dist, dev):
     ev = lambda: torch.cuda.Event()
 
     def one():
-        e_blk = ev()
+        # Layer 0's block rows and queries go first; the other layers' block rows
+        # follow and are spliced while layer 0's attention runs.
+        e_blk0, e_blk = ev(), ev()
         with torch.cuda.stream(s_in):
-            wl.bk.copy_(h_bk, non_blocking=True)
-            wl.bv.copy_(h_bv, non_blocking=True)
-            wl.q_suf.copy_(h_qs, non_blocking=True)
-            e_blk.record(s_in)
-        stream.wait_event(e_blk)
-        nexus.splice_kv(wl.cache, wl.d_pt, wl.h_pt, 2, wl.max_pages, wl.blocks, wl.segs, 0, L,
+            wl.bk[:1].copy_(h_bk[:1], non_blocking=True)
+            wl.bv[:1].copy_(h_bv[:1], non_blocking=True)
+            e_blk0.record(s_in)
+        stream.wait_event(e_blk0)
+        nexus.splice_kv(wl.cache, wl.d_pt, wl.h_pt, 2, wl.max_pages, wl.blocks, wl.segs, 0, 1,
                         stream)
         e_in = [None] * L
         e_done = [None] * L
@@ -943,6 +947,15 @@ def _e2e(wl, stream, args, barrier, world, dist, dev):
                 qbuf[b][0].copy_(h_q[l], non_blocking=True)
                 e_in[l] = ev()
                 e_in[l].record(s_in)
+                if l == 0:
+                    wl.bk[1:].copy_(h_bk[1:], non_blocking=True)
+                    wl.bv[1:].copy_(h_bv[1:], non_blocking=True)
+                    wl.q_suf.copy_(h_qs, non_blocking=True)
+                    e_blk.record(s_in)
+            if l == 1:
+                stream.wait_event(e_blk)
+                nexus.splice_kv(wl.cache, wl.d_pt, wl.h_pt, 2, wl.max_pages, wl.blocks, wl.segs,
+                                1, L, stream)
             stream.wait_event(e_in[l])
             if l >= 2:
                 stream.wait_event(e_out[l - 2])        # O of layer l-2 left obuf[b]
@@ -956,6 +969,7 @@ def _e2e(wl, stream, args, barrier, world, dist, dev):
                 h_o[b].copy_(obuf[b][0], non_blocking=True)
                 e_out[l] = ev()
                 e_out[l].record(s_out)
+        stream.wait_event(e_blk)                       # the suffix's queries (and L = 1)
         for l in range(L):
             nexus.suffix_attention(wl.cache, wl.d_pt, 2, wl.max_pages, [wl.T], [wl.R_split],
                                    wl.q_suf[l:l + 1], wl.o_suf[l:l + 1], wl.lse_suf[l:l + 1], HQ,

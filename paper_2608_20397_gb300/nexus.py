@@ -580,3 +580,26 @@ def host_empty(shape, dtype):
     raw = (ctypes.c_char * max(nbytes, 1)).from_address(m.ptr)
     raw._mapping = m                        # the tensor's storage keeps `raw`, and so `m`, alive
     return torch.frombuffer(raw, dtype=torch.uint8)[:nbytes].view(dtype).view(shape)
+
+
+_GROUP_ALIGN = 1 << 16
+
+
+def host_empty_group(specs):
+    """Several staging tensors, ``[(shape, dtype), ...]``, carved out of ONE
+    nexus_host_alloc mapping at 64 KiB-aligned offsets, in order. Small buffers
+    staged together this way share the huge pages a large mapping gets (a
+    mapping of less than a quarter of the huge page size is made of base pages,
+    from which copies can be many times slower). Returns the tensors as a list;
+    the mapping lives while any of them does."""
+    import torch
+    layout, total = [], 0
+    for shape, dtype in specs:
+        shape = tuple(int(n) for n in shape)
+        nbytes = int(np.prod(shape, dtype=np.int64)) * torch.empty((), dtype=dtype).element_size()
+        layout.append((total, nbytes, shape, dtype))
+        total += -(-nbytes // _GROUP_ALIGN) * _GROUP_ALIGN
+    if not layout:
+        return []
+    base = host_empty((max(total, 1),), torch.uint8)
+    return [base[off:off + n].view(dtype).view(shape) for off, n, shape, dtype in layout]

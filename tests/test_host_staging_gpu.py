@@ -65,3 +65,30 @@ def test_large_staging_region(dev):
     back.copy_(h, non_blocking=True)
     torch.cuda.synchronize()
     assert torch.equal(back.view(torch.int16), d.view(torch.int16))
+
+
+def test_group_of_staging_tensors(dev):
+    """Tensors carved out of one mapping: 64 KiB-aligned, disjoint, each moving
+    its own bytes."""
+    specs = [((3, 7), torch.bfloat16), ((5000,), torch.float32), ((1,), torch.int8),
+             ((48, 64, 40, 128), torch.bfloat16)]
+    ts = nexus.host_empty_group(specs)
+    assert [tuple(t.shape) for t in ts] == [s for s, _ in specs]
+    assert [t.dtype for t in ts] == [d for _, d in specs]
+    starts = [t.data_ptr() for t in ts]
+    assert all(p % 65536 == 0 for p in starts)
+    ends = [p + t.numel() * t.element_size() for p, t in zip(starts, ts)]
+    assert all(ends[i] <= starts[i + 1] for i in range(len(ts) - 1))
+    g = torch.Generator().manual_seed(3)
+    for t in ts:
+        t.copy_(torch.randint(-100, 100, t.shape, generator=g).to(t.dtype))
+    want = [t.clone() for t in ts]
+    d = [t.to(dev, non_blocking=True) for t in ts]
+    torch.cuda.synchronize()                 # the copies have read the host bytes
+    for t in ts:
+        t.zero_()
+    for t, x in zip(ts, d):
+        t.copy_(x, non_blocking=True)
+    torch.cuda.synchronize()
+    assert all(torch.equal(t, w) for t, w in zip(ts, want))
+    assert nexus.host_empty_group([]) == []
