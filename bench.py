@@ -478,9 +478,11 @@ def _profile_only(wl, args, stream):
             qkv_kv, qkv_n, qkv_row = wl.n_past, wl.n_past, 0
         dev = wl.kp.device
         qkv_x = randn_bf16((qkv_n, HIDDEN), 1000, dev)
-        qkv_w, qkv_b = qkv_weights(HQ + 2 * HKV, HIDDEN, 1001, dev)
+        # three layers' weights in turn (220 MB, more than L2), as in the bench line
+        qkv_wbs = [qkv_weights(HQ + 2 * HKV, HIDDEN, 1001 + i, dev) for i in range(3)]
         qkv_q = torch.empty((qkv_n, HQ, D), dtype=torch.bfloat16, device=dev)
         qkv_flops = 2.0 * qkv_n * HIDDEN * (HQ + 2 * HKV) * D
+    launch_no = [0]
 
     if args.profile == "slb":
         # the 1M-tool registry of the bench's large tool scan, one query per launch
@@ -502,6 +504,8 @@ def _profile_only(wl, args, stream):
         if args.profile == "slb":
             nexus.slb_route(slb_t, slb_ts, slb_q, slb_qs, *slb_out, slb_ws, stream=stream)
         elif args.profile == "qkv":
+            qkv_w, qkv_b = qkv_wbs[launch_no[0] % 3]
+            launch_no[0] += 1
             nexus.suffix_qkv(wl.cache, wl.d_pt, 2, wl.max_pages, [qkv_kv], [qkv_n], qkv_x, qkv_w,
                              qkv_b, qkv_q, layer=0, n_q_heads=HQ, rows=[qkv_row], stream=stream)
         elif args.profile == "splice":
@@ -567,22 +571,27 @@ def _profile_only(wl, args, stream):
 def _qkv_measure(wl, stream, peaks, peak_kind, with_oracle, warmup=3, reps=10):
     """Fresh Q, K, V of re-decoded tokens (one layer per launch), timed apart
     from the step: all 32768 tokens of the re-prefill (R = 100 %, Sec. III-C)
-    and the 64-token suffix. Inputs exceed L2 (x alone is 335 MB)."""
+    and the 64-token suffix. Consecutive launches take the weights of different
+    layers, three 73 MB matrices in turn (220 MB, more than L2), as a layer-by-
+    layer re-decode does; the 64-token launch reads its weight from DRAM."""
     import torch
 
     from paper_2608_20397_gb300.workloads import HIDDEN, qkv_weights, randn_bf16
     nexus = wl.nexus
     dev = wl.kp.device
     n_heads = HQ + 2 * HKV
-    w, b = qkv_weights(n_heads, HIDDEN, 1001, dev)
+    wbs = [qkv_weights(n_heads, HIDDEN, 1001 + i, dev) for i in range(3)]
+    w, b = wbs[0]
     x = randn_bf16((wl.n_past, HIDDEN), 1000, dev)
     q = torch.empty((wl.n_past, HQ, D), dtype=torch.bfloat16, device=dev)
     cases = {"reprefill": (wl.n_past, wl.n_past, 0), "suffix": (wl.T, wl.R_split, 1)}
-    out = {"kernel": "qkv_kernel", "hidden": HIDDEN, "heads": f"{HQ} q + {HKV} k + {HKV} v"}
+    out = {"kernel": "qkv_kernel", "hidden": HIDDEN, "heads": f"{HQ} q + {HKV} k + {HKV} v",
+           "weights": "three layers' weights in turn (220 MB > L2)"}
     for name, (kv, n, row) in cases.items():
         def one(l):
-            nexus.suffix_qkv(wl.cache, wl.d_pt, 2, wl.max_pages, [kv], [n], x[:n], w, b, q[:n],
-                             layer=l % wl.L, n_q_heads=HQ, rows=[row], stream=stream)
+            wl_, bl_ = wbs[l % 3]
+            nexus.suffix_qkv(wl.cache, wl.d_pt, 2, wl.max_pages, [kv], [n], x[:n], wl_, bl_,
+                             q[:n], layer=l % wl.L, n_q_heads=HQ, rows=[row], stream=stream)
         for i in range(warmup):
             one(i)
         a = torch.cuda.Event(enable_timing=True)
