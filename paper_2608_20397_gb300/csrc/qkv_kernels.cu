@@ -10,8 +10,8 @@
 // band rather than once per wave. Up to 64 tokens (a short re-decoded suffix)
 // the launch only streams the weight: tiles are one head wide (twice the
 // CTAs), only 64 token rows are copied per box (the products' rows 64-127
-// belong to no token and are never stored), and a stage holds four boxes of
-// consecutive hidden features, so each weight row is read 512 contiguous bytes
+// belong to no token and are never stored), and a stage holds three boxes of
+// consecutive hidden features, so each weight row is read 384 contiguous bytes
 // at a time:
 //   warp 0     TMA producer: X and W tiles of 64 hidden features per stage,
 //              128-byte swizzle, 4-stage ring (48 KiB a stage)
@@ -71,10 +71,12 @@ struct QkvShape {
   static_assert(kSubBytes % 1024 == 0 && kABytes % 1024 == 0, "128-byte swizzle atoms");
 };
 using LongTiles = QkvShape<256, 128, 4, 1>;   // 128 tokens x two heads, 4 stages of 48 KiB
-// Up to 64 tokens x one head: 2 stages of four consecutive 64-feature boxes
-// (96 KiB), so each weight row is read 512 contiguous bytes at a time (one
-// box per stage, 128 bytes per row and stage, ran 44 % slower).
-using ShortTiles = QkvShape<128, 64, 2, 4>;
+// Up to 64 tokens x one head: 3 stages of three consecutive 64-feature boxes
+// (72 KiB), so each weight row is read 384 contiguous bytes at a time and a
+// third stage is in flight while the products consume one (two stages of four
+// boxes: 8 % slower; one box per stage, 128 bytes per row and stage: 23 %
+// slower even with 9 stages).
+using ShortTiles = QkvShape<128, 64, 3, 3>;
 
 __device__ __forceinline__ void record_timeout(volatile int* abort) {
   *abort = 1;
