@@ -185,6 +185,12 @@ constexpr int kSlbSmallQueries = 4;   // up to this many queries: the latency pa
 constexpr int kSlbStreamMinTools = 16384;
 constexpr int kSlbStreamSmemPerCta = 110 * 1024;  // stage ring + queries, two CTAs per SM
 cudaError_t launch_slb(const SlbLaunch& p, int grid, cudaStream_t stream);
+// 5..32 queries over at least kSlbStreamMinTools tools, dim a multiple of 64 up
+// to kSlbTcMaxDim: tensor-core scan; `tools` maps the int8 codes [n_tools][dim]
+// with 64 x 128 boxes.
+constexpr int kSlbTcMaxDim = 1024;
+cudaError_t launch_slb_tc(const SlbLaunch& p, const CUtensorMap& tools, int grid,
+                          cudaStream_t stream);
 cudaError_t slb_take_timeout(unsigned int* flag, cudaStream_t stream);
 
 }  // namespace nexus

@@ -253,6 +253,22 @@ bool encode_2d_sw128(CUtensorMap* m, const void* base, uint64_t inner, uint64_t 
   return r == CUDA_SUCCESS;
 }
 
+// int8 [outer][inner] with boxes of 64 bytes x box_outer rows, no swizzle.
+bool encode_2d_u8(CUtensorMap* m, const void* base, uint64_t inner, uint64_t outer,
+                  uint32_t box_outer) {
+  auto enc = tensor_map_encoder();
+  if (!enc) return false;
+  const cuuint64_t dims[2] = {inner, outer};
+  const cuuint64_t strides[1] = {inner};
+  const cuuint32_t box[2] = {64, box_outer};
+  const cuuint32_t elem[2] = {1, 1};
+  const CUresult r = enc(m, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<void*>(base), dims,
+                         strides, box, elem, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                         CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                         CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
 // Tool scan: CTAs of 8 warps. Few queries (the latency path, 64 registers, 4
 // CTAs per SM): 8 tools per CTA, one per warp, up to four CTAs per SM, so a
 // large registry keeps 32 warps of loads in flight on every SM. Batches (one
@@ -749,6 +765,19 @@ nexus_status nexus_slb_route(const int8_t* d_tools, const float* d_tool_scales, 
     p.top_idx = d_top_idx + 2 * static_cast<int64_t>(q0);
     p.top_score = d_top_score + 2 * static_cast<int64_t>(q0);
     p.route = d_route + q0;
+    if (p.n_queries > kSlbSmallQueries && n_tools >= kSlbStreamMinTools && dim % 64 == 0 &&
+        dim <= kSlbTcMaxDim) {
+      // A batch over a large registry: the exact bf16 tensor-core scan, one CTA
+      // per SM walking tiles of 128 tools.
+      CUtensorMap tmap;
+      if (!encode_2d_u8(&tmap, d_tools, static_cast<uint64_t>(dim),
+                        static_cast<uint64_t>(n_tools), 128))
+        return NEXUS_ECUDA;
+      grid = static_cast<int>(std::min<int64_t>((n_tools + 127) / 128, num_sms()));
+      if (launch_slb_tc(p, tmap, grid, static_cast<cudaStream_t>(stream)) != cudaSuccess)
+        return NEXUS_ECUDA;
+      continue;
+    }
     if (launch_slb(p, grid, static_cast<cudaStream_t>(stream)) != cudaSuccess) return NEXUS_ECUDA;
   }
   return NEXUS_OK;

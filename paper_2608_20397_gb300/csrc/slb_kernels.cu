@@ -8,7 +8,8 @@
 // the tool row (coalesced) and multiplies them with the same words of each query
 // by dp4a. Batches of 5..32 queries (slb_kernel) keep the queries in shared
 // memory and reduce with a 31-shuffle butterfly that leaves lane q with the exact
-// integer dot of query q, so lane q keeps query q's running top two. Up to 4
+// integer dot of query q, so lane q keeps query q's running top two; over large
+// registries they run on the tensor cores instead (slb_tc_kernel, below). Up to 4
 // queries (slb_small_kernel, the routing of single requests) read the query
 // words straight into registers, load all of a tool's words at once and run
 // with one or two tools per warp, for latency; over large registries they
@@ -512,6 +513,290 @@ cudaError_t launch_stream_as(const SlbLaunch& p, int grid, cudaStream_t stream) 
   return cudaGetLastError();
 }
 
+// ---------------------------------------------------------------------------
+// Batches of 5..32 queries over a large registry on the tensor cores. The
+// integer dot products are computed exactly by bf16 products with float32
+// accumulation: every code lies in [-127, 127], which bf16 holds exactly, and
+// for dim <= 1024 every partial sum is an integer of magnitude at most
+// 1024 * 127 * 127 < 2^24, which float32 holds exactly, so the order of the
+// additions does not matter and the scores equal those of the dp4a kernels bit
+// for bit. A CTA walks tiles of 128 tools; per 64-dimension chunk of a tile:
+//   warp 0     TMA copy of the chunk's int8 codes (128 x 64 bytes) into an
+//              8-stage ring
+//   warps 2-5  convert the codes to bf16 in the 128-byte-swizzled K-major
+//              layout of the MMA's A operand (4-slot ring): a code v becomes
+//              the float 2^23 + (v + 128), minus 2^23 + 128, packed to bf16
+//   warp 1     tcgen05.mma 128 x 32 x 16 against the queries (bf16, resident,
+//              rows past the batch zero), four per chunk, into one of two
+//              32-column TMEM accumulators
+//   warps 6-9  read the accumulator (thread = tool), scale, and keep per-query
+//              top twos through a shared-memory transpose
+// Every wait is bounded; on expiry the CTA records a timeout and winds down.
+constexpr int kTcThreads = 320;
+constexpr int kTcTools = 128;
+constexpr int kTcStaging = 8;                  // int8 chunk ring
+constexpr int kTcASlots = 4;                   // bf16 A ring
+constexpr uint32_t kTcStBytes = kTcTools * 64;        // 8 KiB
+constexpr uint32_t kTcABytes = kTcTools * 128;        // 16 KiB
+constexpr uint32_t kTcOffB = 0;                       // queries: dim / 64 chunks of 4 KiB
+constexpr uint32_t kTcOffSt = 64 * 1024;
+constexpr uint32_t kTcOffA = kTcOffSt + kTcStaging * kTcStBytes;
+constexpr uint32_t kTcOffSc = kTcOffA + kTcASlots * kTcABytes;   // scores [128][33]
+constexpr uint32_t kTcOffTop = kTcOffSc + kTcTools * 33 * 4;
+constexpr uint32_t kTcOffQs = kTcOffTop + 4 * 32 * sizeof(Top2);
+constexpr uint32_t kTcOffBar = kTcOffQs + 32 * 4;
+constexpr int kTcBars = 2 * kTcStaging + 2 * kTcASlots + 4 + 1;
+constexpr uint32_t kTcOffMisc = kTcOffBar + kTcBars * 8;
+constexpr uint32_t kTcSmem = kTcOffMisc + 32 + 1024;
+static_assert(kTcSmem <= 227 * 1024, "shared memory budget");
+constexpr uint64_t kTcBudgetNs = 2000000000ull;
+constexpr uint64_t kTcDrainNs = 200000000ull;
+
+__device__ __forceinline__ void record_timeout(volatile int* abort) {
+  *abort = 1;
+  atomicOr(&g_slb_timeout, 1u);
+}
+
+// 16 codes -> 16 bf16 (8 words), exactly.
+__device__ __forceinline__ void codes_to_bf16(const uint4& c, uint32_t (&o)[8]) {
+  const uint32_t w[4] = {c.x, c.y, c.z, c.w};
+  // __byte_perm selector 0x765k: byte k of u, then bytes 1-3 of 0x4B000000
+  const float off = 8388736.f;   // 2^23 + 128
+#pragma unroll
+  for (int k = 0; k < 4; ++k) {
+    const uint32_t u = w[k] ^ 0x80808080u;   // bytes v + 128
+    const float f0 = __uint_as_float(__byte_perm(u, 0x4B000000u, 0x7650)) - off;
+    const float f1 = __uint_as_float(__byte_perm(u, 0x4B000000u, 0x7651)) - off;
+    const float f2 = __uint_as_float(__byte_perm(u, 0x4B000000u, 0x7652)) - off;
+    const float f3 = __uint_as_float(__byte_perm(u, 0x4B000000u, 0x7653)) - off;
+    o[2 * k] = pack_bf16x2(f0, f1);
+    o[2 * k + 1] = pack_bf16x2(f2, f3);
+  }
+}
+
+__device__ __forceinline__ void named_sync_128(int id) {
+  asm volatile("bar.sync %0, 128;" ::"r"(id) : "memory");
+}
+
+__global__ void __launch_bounds__(kTcThreads, 1)
+slb_tc_kernel(const __grid_constant__ SlbLaunch p, const __grid_constant__ CUtensorMap tmap) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~static_cast<uintptr_t>(1023));
+  const uint32_t sbase = smem_u32(smem);
+  auto bar = [&](int i) -> uint32_t { return sbase + kTcOffBar + 8u * i; };
+  const int B_FST = 0, B_EST = kTcStaging, B_FA = 2 * kTcStaging, B_EA = B_FA + kTcASlots,
+            B_AF = B_EA + kTcASlots, B_AE = B_AF + 2, B_FIN = B_AE + 2;
+  volatile uint32_t* tmem_slot = reinterpret_cast<volatile uint32_t*>(smem + kTcOffMisc);
+  volatile int* abort = reinterpret_cast<volatile int*>(smem + kTcOffMisc + 4);
+  volatile int* never = reinterpret_cast<volatile int*>(smem + kTcOffMisc + 8);
+  volatile int* last = reinterpret_cast<volatile int*>(smem + kTcOffMisc + 12);
+  float* s_sc = reinterpret_cast<float*>(smem + kTcOffSc);
+  Top2* s_top = reinterpret_cast<Top2*>(smem + kTcOffTop);
+  float* s_qs = reinterpret_cast<float*>(smem + kTcOffQs);
+  const volatile unsigned int* gabort = &g_slb_timeout;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int nq = p.n_queries;
+  const int n_chunks = p.dim / 64;
+  const int n_tiles = (p.n_tools + kTcTools - 1) / kTcTools;
+
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < kTcBars; ++i) {
+      uint32_t count = 1;
+      if ((i >= B_EST && i < B_EST + kTcStaging) || (i >= B_FA && i < B_FA + kTcASlots) ||
+          (i >= B_AE && i < B_AE + 2))
+        count = 4;   // one arrival per converter / epilogue warp
+      mbar_init(bar(i), count);
+    }
+    *abort = 0;
+    *never = 0;
+    fence_mbar_init();
+  }
+  if (threadIdx.x < 32) s_qs[threadIdx.x] = threadIdx.x < nq ? p.query_scales[threadIdx.x] : 0.f;
+  // queries -> bf16 B operand: chunk c holds rows 0..31 (queries; zero past the batch)
+  for (int i = threadIdx.x; i < n_chunks * 32 * 4; i += kTcThreads) {
+    const int c = i / 128, row = (i / 4) % 32, q16 = i % 4;
+    uint4 v = make_uint4(0, 0, 0, 0);
+    if (row < nq)
+      v = *reinterpret_cast<const uint4*>(p.queries + (int64_t)row * p.dim + c * 64 + q16 * 16);
+    uint32_t o[8];
+    codes_to_bf16(v, o);
+    const uint32_t rb = sbase + kTcOffB + c * 4096 + row * 128;
+    st_shared_v4(rb + (((2 * q16) ^ (row & 7)) << 4), o[0], o[1], o[2], o[3]);
+    st_shared_v4(rb + (((2 * q16 + 1) ^ (row & 7)) << 4), o[4], o[5], o[6], o[7]);
+  }
+  fence_proxy_async_smem();
+  if (warp == 1) {
+    tmem_alloc(sbase + kTcOffMisc, 64);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  if (warp == 0) {
+    // ------------------------------------------------------ TMA producer
+    if (lane == 0) {
+      prefetch_tmap(&tmap);
+      int it = 0;
+      bool ok = true;
+      for (int t = blockIdx.x; t < n_tiles && ok; t += gridDim.x) {
+        for (int c = 0; c < n_chunks; ++c, ++it) {
+          const int s = it % kTcStaging;
+          if (it >= kTcStaging &&
+              !mbar_wait(bar(B_EST + s), ((it / kTcStaging) - 1) & 1, kTcBudgetNs, abort, gabort)) {
+            ok = false;
+            record_timeout(abort);
+            break;
+          }
+          mbar_arrive_expect_tx(bar(B_FST + s), kTcStBytes);
+          tma_load_2d(sbase + kTcOffSt + s * kTcStBytes, &tmap, bar(B_FST + s), c * 64,
+                      t * kTcTools);
+        }
+      }
+      for (int i = max(0, it - kTcStaging); i < it; ++i)
+        mbar_wait(bar(B_FST + i % kTcStaging), (i / kTcStaging) & 1, kTcDrainNs, never);
+    }
+    __syncwarp();
+  } else if (warp == 1) {
+    // ------------------------------------------------------ MMA issuer
+    if (lane == 0) {
+      constexpr uint32_t idesc = idesc_bf16_f32(kTcTools, 32, false);
+      const uint64_t da0 = smem_desc(sbase + kTcOffA, 16, 1024, kSwizzle128B);
+      const uint64_t db0 = smem_desc(sbase + kTcOffB, 16, 1024, kSwizzle128B);
+      int it = 0, acc_it = 0;
+      bool ok = true;
+      for (int t = blockIdx.x; t < n_tiles && ok; t += gridDim.x, ++acc_it) {
+        const int b = acc_it & 1;
+        if (acc_it >= 2 &&
+            !mbar_wait(bar(B_AE + b), ((acc_it >> 1) - 1) & 1, kTcBudgetNs, abort, gabort)) {
+          ok = false;
+          record_timeout(abort);
+          break;
+        }
+        tc_fence_after();
+        for (int c = 0; c < n_chunks; ++c, ++it) {
+          const int a = it % kTcASlots;
+          if (!mbar_wait(bar(B_FA + a), (it / kTcASlots) & 1, kTcBudgetNs, abort, gabort)) {
+            ok = false;
+            record_timeout(abort);
+            break;
+          }
+          tc_fence_after();
+#pragma unroll
+          for (int kk = 0; kk < 4; ++kk)
+            mma_bf16(tmem + b * 32, da0 + ((a * kTcABytes + kk * 32) >> 4),
+                     db0 + ((c * 4096 + kk * 32) >> 4), idesc, (c | kk) != 0 ? 1u : 0u);
+          mma_commit(bar(B_EA + a));
+        }
+        if (ok) mma_commit(bar(B_AF + b));
+      }
+      mma_commit(bar(B_FIN));
+      mbar_wait(bar(B_FIN), 0, kTcDrainNs, never);
+    }
+    __syncwarp();
+  } else if (warp < 6) {
+    // ------------------------------------------------------ converters
+    const int ct = threadIdx.x - 64;
+    int it = 0;
+    bool ok = true;
+    for (int t = blockIdx.x; t < n_tiles && ok; t += gridDim.x) {
+      for (int c = 0; c < n_chunks; ++c, ++it) {
+        const int s = it % kTcStaging, a = it % kTcASlots;
+        bool w = mbar_wait(bar(B_FST + s), (it / kTcStaging) & 1, kTcBudgetNs, abort, gabort);
+        if (w && it >= kTcASlots)
+          w = mbar_wait(bar(B_EA + a), ((it / kTcASlots) - 1) & 1, kTcBudgetNs, abort, gabort);
+        ok = __all_sync(0xffffffffu, w);
+        if (!ok) {
+          if (lane == 0) record_timeout(abort);
+          break;
+        }
+        const uint8_t* st = smem + kTcOffSt + s * kTcStBytes;
+        const uint32_t ab = sbase + kTcOffA + a * kTcABytes;
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+          const int i = ct + 128 * k, row = i >> 2, q16 = i & 3;
+          const uint4 v = *reinterpret_cast<const uint4*>(st + row * 64 + q16 * 16);
+          uint32_t o[8];
+          codes_to_bf16(v, o);
+          st_shared_v4(ab + row * 128 + (((2 * q16) ^ (row & 7)) << 4), o[0], o[1], o[2], o[3]);
+          st_shared_v4(ab + row * 128 + (((2 * q16 + 1) ^ (row & 7)) << 4), o[4], o[5], o[6], o[7]);
+        }
+        fence_proxy_async_smem();
+        __syncwarp();
+        if (lane == 0) {
+          mbar_arrive(bar(B_EST + s));
+          mbar_arrive(bar(B_FA + a));
+        }
+      }
+    }
+  } else {
+    // ------------------------------------------------------ epilogue
+    const int quad = warp & 3;                  // TMEM lanes [32 quad, 32 quad + 32)
+    const int r = quad * 32 + lane;             // this thread's tool row of the tile
+    const int et = threadIdx.x - 192;
+    const int q = et & 31, part = et >> 5;      // transposed role: query q, rows of `part`
+    const uint32_t lane_base = static_cast<uint32_t>(quad * 32) << 16;
+    Top2 top = empty_top2();
+    bool ok = true;
+    int acc_it = 0;
+    for (int t = blockIdx.x; t < n_tiles; t += gridDim.x, ++acc_it) {
+      const int b = acc_it & 1;
+      if (ok) {
+        const bool w = mbar_wait(bar(B_AF + b), (acc_it >> 1) & 1, kTcBudgetNs, abort, gabort);
+        ok = __all_sync(0xffffffffu, w);
+        if (!ok && lane == 0) record_timeout(abort);
+      }
+      if (ok) {
+        tc_fence_after();
+        uint32_t v[32];
+        tmem_ld32(tmem + lane_base + b * 32, v);
+        tmem_ld_wait();
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(bar(B_AE + b));
+        const int tool = t * kTcTools + r;
+        const float st = tool < p.n_tools ? __ldg(p.tool_scales + tool) : 0.f;
+#pragma unroll
+        for (int j = 0; j < 32; ++j) s_sc[r * 33 + j] = __uint_as_float(v[j]) * (s_qs[j] * st);
+      }
+      named_sync_128(1);
+      if (ok && q < nq) {
+        const int row0 = part * 32;
+        const int n_valid = min(32, p.n_tools - (t * kTcTools + row0));
+        for (int rr = 0; rr < n_valid; ++rr)
+          push(top, s_sc[(row0 + rr) * 33 + q], t * kTcTools + row0 + rr);
+      }
+      named_sync_128(1);
+    }
+    s_top[part * 32 + q] = top;
+    named_sync_128(1);
+    if (part == 0 && q < nq) {
+      Top2 m = s_top[q];
+      for (int w = 1; w < 4; ++w) {
+        const Top2 o = s_top[w * 32 + q];
+        push(m, o.s1, o.i1);
+        push(m, o.s2, o.i2);
+      }
+      const int64_t k = (int64_t)blockIdx.x * 32 + q;
+      p.part_score[2 * k] = m.s1;
+      p.part_score[2 * k + 1] = m.s2;
+      p.part_idx[2 * k] = m.i1;
+      p.part_idx[2 * k + 1] = m.i2;
+      __threadfence();
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  if (warp == 1) tmem_dealloc(tmem, 64);
+  if (threadIdx.x == 0) *last = atomicAdd(p.counter, 1u) == gridDim.x - 1;
+  __syncthreads();
+  if (*last && warp < kSlbWarps) final_merge(p, warp, lane);
+}
+
 template <int kQ>
 cudaError_t launch_slb_as(const SlbLaunch& p, int grid, cudaStream_t stream) {
   const size_t smem = (size_t)kQ * p.dim;
@@ -548,6 +833,16 @@ cudaError_t launch_slb(const SlbLaunch& p, int grid, cudaStream_t stream) {
   if (p.n_queries <= 8) return launch_slb_as<8>(p, grid, stream);
   if (p.n_queries <= 16) return launch_slb_as<16>(p, grid, stream);
   return launch_slb_as<32>(p, grid, stream);
+}
+
+cudaError_t launch_slb_tc(const SlbLaunch& p, const CUtensorMap& tools, int grid,
+                          cudaStream_t stream) {
+  if (p.n_queries <= 0 || grid <= 0) return cudaSuccess;
+  cudaError_t e = cudaFuncSetAttribute(slb_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       (int)kTcSmem);
+  if (e != cudaSuccess) return e;
+  slb_tc_kernel<<<(unsigned)grid, kTcThreads, kTcSmem, stream>>>(p, tools);
+  return cudaGetLastError();
 }
 
 cudaError_t slb_take_timeout(unsigned int* flag, cudaStream_t stream) {

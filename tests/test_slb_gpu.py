@@ -169,3 +169,28 @@ def test_slb_streamed_workspace_reuse(dev):
     for a, b in zip(first, second):
         assert np.array_equal(a, b)
     assert not ws[:16].any()
+
+
+@pytest.mark.parametrize("dim,n_tools,nq", [(768, 16384 + 37, 5), (64, 20000 + 3, 32),
+                                            (1024, 16384, 17), (512, 100_003, 8),
+                                            (1088, 16384, 8)])
+def test_slb_tensor_core_batches(dev, dim, n_tools, nq):
+    # Batches of 5..32 queries over 16384 tools and more, dim a multiple of 64 up
+    # to 1024, are scanned by bf16 products on the tensor cores: exact integer dots
+    # (|partial sums| <= 1024 * 127^2 < 2^24), so exact parity. Rows of +-127 reach
+    # that bound; a three-way tie, a zero scale and a partial last tile of 128
+    # tools are planted. dim 1088 is past the bound and keeps the dp4a scan.
+    r = np.random.default_rng(dim + n_tools + nq)
+    tc = r.integers(-127, 128, (n_tools, dim), dtype=np.int8)
+    ts = (r.random(n_tools, dtype=np.float32) * np.float32(0.01)).astype(np.float32)
+    qc = r.integers(-127, 128, (nq, dim), dtype=np.int8)
+    qs = (r.random(nq, dtype=np.float32) * np.float32(0.01)).astype(np.float32)
+    tc[11], tc[12] = 127, -127
+    qc[0], qc[1] = 127, -127
+    ts[13] = 0.0
+    tc[2] = tc[3]
+    tc[n_tools - 1] = tc[3]
+    ts[2] = ts[n_tools - 1] = ts[3]
+    got = run(dev, tc, ts, qc, qs)
+    assert nexus.device_status() == nexus.OK
+    check(got, tc, ts, qc, qs)
