@@ -863,7 +863,7 @@ def _slb_measure(wl, stream, peaks, peak_kind, with_oracle, reps=200):
                                  "decision copied out, through the Python binding"},
            "large": {"tools": n_big, "dim": dim, "by_batch": by_batch,
                      "note": "8 and 32 queries per launch: exact bf16 tensor-core scan "
-                             "(slb_tc_kernel), flat in the batch size at ~2.3 TB/s"},
+                             "(slb_tc_kernel), flat in the batch size at ~2.5 TB/s"},
            "roofline": {"bound": "hbm", "kernel": "slb_stream_kernel (1M x 768 codes, 1 query)",
                         "achieved": gbs, "peak": peaks["hbm_gbs"], "unit": "GB/s",
                         "frac": gbs / peaks["hbm_gbs"], "peak_kind": f"copy, {peak_kind}",
