@@ -317,6 +317,8 @@ def main():
                     help="workload of --profile runs (c3: token-innermost V cache)")
     ap.add_argument("--tokens", type=int, default=0,
                     help="--profile qkv: re-decode this many last tokens of the spliced cache")
+    ap.add_argument("--queries", type=int, default=1,
+                    help="--profile slb: queries per launch (1..32)")
     args = ap.parse_args()
 
     rank = int(os.environ.get("RANK", "0"))
@@ -492,13 +494,14 @@ def _profile_only(wl, args, stream):
         slb_t = torch.randint(-127, 128, (1 << 20, 768), generator=g, device=dev,
                               dtype=torch.int32).to(torch.int8)
         slb_ts = torch.rand(1 << 20, generator=g, device=dev) * 0.01
-        slb_q = torch.randint(-127, 128, (1, 768), generator=g, device=dev,
+        nq = max(1, min(32, args.queries))
+        slb_q = torch.randint(-127, 128, (nq, 768), generator=g, device=dev,
                               dtype=torch.int32).to(torch.int8)
-        slb_qs = torch.rand(1, generator=g, device=dev) * 0.01
+        slb_qs = torch.rand(nq, generator=g, device=dev) * 0.01
         slb_ws = torch.zeros(nexus.slb_workspace_size(1 << 20), dtype=torch.uint8, device=dev)
-        slb_out = (torch.empty((1, 2), dtype=torch.int32, device=dev),
-                   torch.empty((1, 2), dtype=torch.float32, device=dev),
-                   torch.empty(1, dtype=torch.int32, device=dev))
+        slb_out = (torch.empty((nq, 2), dtype=torch.int32, device=dev),
+                   torch.empty((nq, 2), dtype=torch.float32, device=dev),
+                   torch.empty(nq, dtype=torch.int32, device=dev))
 
     def one():
         if args.profile == "slb":
@@ -543,7 +546,8 @@ def _profile_only(wl, args, stream):
     ms = a.elapsed_time(b) / args.steps
     if args.profile == "slb":
         gbs = (1 << 20) * 772.0 / (ms * 1e-3) / 1e9
-        print(json.dumps({"profile": "slb", "tools": 1 << 20, "ms_per_launch": ms,
+        print(json.dumps({"profile": "slb", "tools": 1 << 20, "queries": args.queries,
+                          "ms_per_launch": ms,
                           "rate": f"{gbs:.1f} GB/s", "status": nexus.status_string(st)}),
               flush=True)
         if st != nexus.OK:
