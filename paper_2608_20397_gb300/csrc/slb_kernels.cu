@@ -8,7 +8,8 @@
 // the tool row (coalesced) and multiplies them with the same words of each query
 // by dp4a. Batches of 5..32 queries (slb_kernel) keep the queries in shared
 // memory and reduce with a 31-shuffle butterfly that leaves lane q with the exact
-// integer dot of query q, so lane q keeps query q's running top two. Up to 4
+// integer dot of query q, so lane q keeps query q's running top two; over large
+// registries they run on the tensor cores instead (slb_tc_kernel, below). Up to 4
 // queries (slb_small_kernel, the routing of single requests) read the query
 // words straight into registers, load all of a tool's words at once and run
 // with one or two tools per warp, for latency; over large registries they
@@ -522,18 +523,19 @@ cudaError_t launch_stream_as(const SlbLaunch& p, int grid, cudaStream_t stream) 
 // for bit. A CTA walks tiles of 128 tools; per 64-dimension chunk of a tile:
 //   warp 0     TMA copy of the chunk's int8 codes (128 x 64 bytes) into an
 //              8-stage ring
-//   warps 2-9  convert the codes to bf16 in the 128-byte-swizzled K-major
+//   warps 2-4, 6-8, 10-11
+//              convert the codes to bf16 in the 128-byte-swizzled K-major
 //              layout of the MMA's A operand (4-slot ring): a code v becomes
 //              the float 2^23 + (v + 128), minus 2^23 + 128, packed to bf16
-//              (two warps per sub-partition, so one's waits hide behind the
-//              other's arithmetic)
+//              (eight warps, none on the issuing thread's sub-partition; warps
+//              5 and 9 stay idle)
 //   warp 1     tcgen05.mma 128 x 32 x 16 against the queries (bf16, resident,
 //              rows past the batch zero), four per chunk, into one of two
 //              32-column TMEM accumulators
-//   warps 10-13 read the accumulator (thread = tool), scale, and keep per-query
+//   warps 12-15 read the accumulator (thread = tool), scale, and keep per-query
 //              top twos through a shared-memory transpose
 // Every wait is bounded; on expiry the CTA records a timeout and winds down.
-constexpr int kTcThreads = 448;
+constexpr int kTcThreads = 512;
 constexpr int kTcTools = 128;
 constexpr int kTcStaging = 8;                  // int8 chunk ring
 constexpr int kTcASlots = 4;                   // bf16 A ring
@@ -697,9 +699,12 @@ slb_tc_kernel(const __grid_constant__ SlbLaunch p, const __grid_constant__ CUten
       mbar_wait(bar(B_FIN), 0, kTcDrainNs, never);
     }
     __syncwarp();
-  } else if (warp < 10) {
+  } else if (warp < 12 && (warp & 3) != 1) {
     // ------------------------------------------------------ converters
-    const int ct = threadIdx.x - 64;
+    // converters sit on warps 2, 3, 4, 6, 7, 8, 10, 11: none shares the issuing
+    // thread's sub-partition (warps 5 and 9 stay idle)
+    const int cw = warp - 2 - (warp > 5 ? 1 : 0) - (warp > 9 ? 1 : 0);
+    const int ct = cw * 32 + lane;
     int it = 0;
     bool ok = true;
     for (int t = blockIdx.x; t < n_tiles && ok; t += gridDim.x) {
@@ -732,11 +737,11 @@ slb_tc_kernel(const __grid_constant__ SlbLaunch p, const __grid_constant__ CUten
         }
       }
     }
-  } else {
+  } else if (warp >= 12) {
     // ------------------------------------------------------ epilogue
     const int quad = warp & 3;                  // TMEM lanes [32 quad, 32 quad + 32)
     const int r = quad * 32 + lane;             // this thread's tool row of the tile
-    const int et = threadIdx.x - 320;
+    const int et = threadIdx.x - 384;
     const int q = et & 31, part = et >> 5;      // transposed role: query q, rows of `part`
     const uint32_t lane_base = static_cast<uint32_t>(quad * 32) << 16;
     Top2 top = empty_top2();
