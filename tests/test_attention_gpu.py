@@ -128,6 +128,18 @@ def test_max_sequences_per_call():
         _check(ks, vs, q, o, lse, kv, ql, 5, what=f"512 sequences, split {split}")
 
 
+def test_split_kv_uneven_pairs():
+    """Automatic split over sequences whose tile pairs differ (full pairs, a
+    sequence of one tile, pairs with a one-tile tail) and an empty sequence in
+    between; every row against the oracle."""
+    kv, ql = [9000, 5000, 7000, 300], [64, 0, 25, 50]
+    cache, d_pt, mp, ks, vs, q = _direct_case(kv, ql, seed=17)
+    _, splits = nexus.attention_workspace_size(kv, ql, 40, 8, 1, 0)
+    assert splits > 1
+    o, lse = _run(cache, d_pt, mp, kv, ql, q, 40, 1, split_kv=0)
+    _check(ks, vs, q, o, lse, kv, ql, 5, what="uneven pairs")
+
+
 def test_reprefill_equals_textbook_causal():
     T = 600
     cache, d_pt, mp, ks, vs, q = _direct_case([T], [T], seed=13)
