@@ -53,8 +53,9 @@ def slb_quantize(x) -> Tuple[np.ndarray, np.ndarray]:
 
 def slb_scores(q_codes, q_scales, t_codes, t_scales) -> np.ndarray:
     """float32 scores [n_queries][n_tools] of the rule above."""
-    # Integer dot products: every product and partial sum is an integer below
-    # 2^24, so a float64 matrix product computes them exactly.
+    # Integer dot products: every product and partial sum is an integer of
+    # magnitude at most 4096 * 128^2 = 2^26, far below 2^53, so a float64 matrix
+    # product computes them exactly.
     qc = np.asarray(q_codes, dtype=np.float64)
     tc = np.asarray(t_codes, dtype=np.float64)
     dots = qc @ tc.T

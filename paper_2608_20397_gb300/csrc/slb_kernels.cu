@@ -516,9 +516,9 @@ cudaError_t launch_stream_as(const SlbLaunch& p, int grid, cudaStream_t stream) 
 // ---------------------------------------------------------------------------
 // Batches of 5..32 queries over a large registry on the tensor cores. The
 // integer dot products are computed exactly by bf16 products with float32
-// accumulation: every code lies in [-127, 127], which bf16 holds exactly, and
-// for dim <= 1024 every partial sum is an integer of magnitude at most
-// 1024 * 127 * 127 < 2^24, which float32 holds exactly, so the order of the
+// accumulation: every int8 code (-128 included) is exact in bf16, and for
+// dim <= 1024 every partial sum is an integer of magnitude at most
+// 1024 * 128 * 128 = 2^24, which float32 holds exactly, so the order of the
 // additions does not matter and the scores equal those of the dp4a kernels bit
 // for bit. A CTA walks tiles of 128 tools; per 64-dimension chunk of a tile:
 //   warp 0     TMA copy of the chunk's int8 codes (128 x 64 bytes) into an

@@ -177,16 +177,17 @@ def test_slb_streamed_workspace_reuse(dev):
 def test_slb_tensor_core_batches(dev, dim, n_tools, nq):
     # Batches of 5..32 queries over 16384 tools and more, dim a multiple of 64 up
     # to 1024, are scanned by bf16 products on the tensor cores: exact integer dots
-    # (|partial sums| <= 1024 * 127^2 < 2^24), so exact parity. Rows of +-127 reach
-    # that bound; a three-way tie, a zero scale and a partial last tile of 128
-    # tools are planted. dim 1088 is past the bound and keeps the dp4a scan.
+    # (|partial sums| <= 1024 * 128^2 = 2^24), so exact parity. Rows of 127 and
+    # -128 reach that bound (tool 12 with query 1: 2^24 at dim 1024); a three-way
+    # tie, a zero scale and a partial last tile of 128 tools are planted. dim
+    # 1088 is past the bound and keeps the dp4a scan.
     r = np.random.default_rng(dim + n_tools + nq)
     tc = r.integers(-127, 128, (n_tools, dim), dtype=np.int8)
     ts = (r.random(n_tools, dtype=np.float32) * np.float32(0.01)).astype(np.float32)
     qc = r.integers(-127, 128, (nq, dim), dtype=np.int8)
     qs = (r.random(nq, dtype=np.float32) * np.float32(0.01)).astype(np.float32)
-    tc[11], tc[12] = 127, -127
-    qc[0], qc[1] = 127, -127
+    tc[11], tc[12] = 127, -128
+    qc[0], qc[1] = 127, -128
     ts[13] = 0.0
     tc[2] = tc[3]
     tc[n_tools - 1] = tc[3]
