@@ -905,6 +905,30 @@ def _profiled_traffic(kernel: str):
         return None
 
 
+def _huge_page_fraction(tensors):
+    """Fraction of the bytes of the mappings that hold these host tensors that
+    the kernel backs with transparent huge pages (Linux /proc/self/smaps), or
+    None where that cannot be read. Copies from page-locked memory on scattered
+    base pages run several times slower, so this explains a slow e2e line."""
+    spans = [(t.data_ptr(), t.data_ptr() + t.numel() * t.element_size()) for t in tensors]
+    try:
+        size = huge = 0
+        cur = None
+        with open("/proc/self/smaps") as f:
+            for line in f:
+                head = line.split()[0]
+                if "-" in head and not head.endswith(":"):
+                    lo, hi = (int(x, 16) for x in head.split("-"))
+                    cur = any(a < hi and lo < b for a, b in spans)
+                elif cur and head == "Size:":
+                    size += int(line.split()[1])
+                elif cur and head == "AnonHugePages:":
+                    huge += int(line.split()[1])
+        return huge / size if size else None
+    except (OSError, ValueError):
+        return None
+
+
 def _e2e(wl, stream, args, barrier, world, dist, dev):
     """The same step through the C ABI with host buffers: every step copies the
     block K/V and every layer's Q in from pinned host memory and reads every
@@ -1008,7 +1032,8 @@ def _e2e(wl, stream, args, barrier, world, dist, dev):
     flops = wl.flops_pre + wl.flops_suf
     return {"value": job_throughput(flops, world, per * 1e3), "unit": "TFLOP/s",
             "ms_per_step": per * 1e3, "h2d_bytes_per_step": int(h2d),
-            "d2h_bytes_per_step": int(d2h)}
+            "d2h_bytes_per_step": int(d2h),
+            "staging_huge_page_fraction": _huge_page_fraction([h_qall, h_oall, h_bk])}
 
 
 if __name__ == "__main__":

@@ -513,8 +513,10 @@ nexus_status nexus_suffix_attention_noalloc(const nexus_kv_cache* cache,
  * this library. The library maps `bytes` of fresh anonymous memory, faults it
  * in and registers it with the CUDA driver, so cudaMemcpyAsync from or to it is
  * asynchronous. Requests of at least a quarter of the kernel's transparent huge
- * page size are rounded up to whole huge pages, aligned to them and advised to
- * use them; smaller ones are rounded up to the base page size. On Grace hosts
+ * page size are rounded up to whole huge pages, aligned to them, advised to use
+ * them and, once faulted in, offered for collapse into huge pages (where the
+ * kernel supports it; both are best effort); smaller ones are rounded up to the
+ * base page size. On Grace hosts
  * (64 KiB base pages, 512 MiB huge pages) copies from page-locked memory on
  * scattered base pages, whether from cudaHostAlloc or registered, ran at 4 to
  * 200 GB/s depending on the buffer; from huge pages at a steady 200 GB/s.

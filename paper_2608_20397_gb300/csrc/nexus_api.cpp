@@ -864,6 +864,13 @@ nexus_status nexus_host_alloc(size_t bytes, void** out) {
   // Fault every page in (zero-filled) before the driver pins them.
   const size_t base = host_base_page();
   for (size_t off = 0; off < len; off += base) static_cast<volatile uint8_t*>(p)[off] = 0;
+  if (extra) {
+    // Where the faults fell back to base pages (memory too fragmented at that
+    // moment), ask the kernel to collapse the range into huge pages now (Linux
+    // 6.1 and later; best effort, an older kernel or a refusal changes nothing).
+    constexpr int kMadvCollapse = 25;
+    madvise(p, len, kMadvCollapse);
+  }
   if (cudaHostRegister(p, len, cudaHostRegisterDefault) != cudaSuccess) {
     cudaGetLastError();
     munmap(p, len);
