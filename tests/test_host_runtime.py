@@ -6,6 +6,7 @@ import re
 from fractions import Fraction
 
 import numpy as np
+import torch
 import pytest
 
 import oracle
@@ -313,6 +314,28 @@ def test_workspace_size_and_split_choice():
     assert s == 1 and n == 0
     assert nexus.attention_workspace_size([10] * 513, [1] * 513, 40, 8, 1, 1) == (0, 0)
     assert nexus.attention_workspace_size([10], [11], 40, 8, 1, 1) == (0, 0)
+
+
+def test_zero_work_calls_succeed_before_any_launch():
+    """Calls with nothing to compute return OK after validation and before any
+    launch or memory access (the FAKE pointers are never dereferenced)."""
+    c = _cache()
+    nexus.suffix_attention(c, FAKE, 2, 8, [10, 50], [0, 0], FAKE, FAKE, stream=0)
+    nexus.suffix_attention(c, FAKE, 2, 8, [10, 50], [0, 0], FAKE, FAKE, split_kv=0, stream=0)
+    nexus.reprefill(c, FAKE, 1, 8, [0], FAKE, FAKE, stream=0)
+    nexus.suffix_attention(c, FAKE, 1, 8, [10], [5], FAKE, FAKE, layer_begin=1, layer_end=1,
+                           stream=0)
+    nexus.suffix_qkv(c, FAKE, 2, 8, [10, 3], [0, 0], FAKE, FAKE, None, FAKE, hidden=64, stream=0)
+    tools = torch.zeros((16, 64), dtype=torch.int8)
+    nexus.slb_route(tools, torch.zeros(16), torch.zeros((0, 64), dtype=torch.int8),
+                    torch.zeros(0), torch.zeros((0, 2), dtype=torch.int32), torch.zeros((0, 2)),
+                    torch.zeros(0, dtype=torch.int32), torch.zeros(16, dtype=torch.uint8),
+                    stream=0)
+    blk = [nexus.block(FAKE, FAKE, 8, 0, 2)]
+    pts = np.array([[0, 1, 2, 3], [4, 5, 6, 7]], np.int32)
+    nexus.splice_kv(c, FAKE, pts, 2, 4, blk, [], 0, 2, stream=0)
+    nexus.splice_kv(c, FAKE, pts, 2, 4, blk, [(nexus.SRC_BLOCK, 0, 0, 0, 0, 8, 0, 0)], 1, 1,
+                    stream=0)
 
 
 def test_attention_rejects_more_than_512_sequences():
