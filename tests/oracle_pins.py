@@ -272,6 +272,35 @@ def pin_attention_library(attention):
             assert np.max(np.abs(o - oc.permute(1, 0, 2).numpy())) < 1e-12
 
 
+def pin_suffix_positions(suffix_positions):
+    """The re-decoded suffix is the trailing R tokens of a T-token cache (Sec. III-C,
+    Sec. V-A): one position per token, R = T is the whole prefill and R = 0 is empty.
+    Through torch's library attention: the queries at these positions, each seeing the
+    keys at or before its position, give the last R rows of the library's built-in
+    causal prefill of all T tokens, which never sees the positions."""
+    for T in (1, 2, 9, 300):
+        assert np.array_equal(np.asarray(suffix_positions(T, T)), np.arange(T))
+        assert len(suffix_positions(T, 0)) == 0
+        for R in sorted({1, 2, T // 2, T - 1, T} - {0}):
+            pos = np.asarray(suffix_positions(T, R))
+            assert pos.shape == (R,)
+            assert pos[-1] == T - 1
+            assert np.all(np.diff(pos) == 1)
+    r = _rs(22)
+    T, Hkv, group, d = 23, 2, 3, 16
+    q = r.standard_normal((T, Hkv * group, d))
+    k = r.standard_normal((T, Hkv, d))
+    v = r.standard_normal((T, Hkv, d))
+    qt = torch.from_numpy(q).permute(1, 0, 2)
+    kt = torch.from_numpy(k).permute(1, 0, 2).repeat_interleave(group, 0)
+    vt = torch.from_numpy(v).permute(1, 0, 2).repeat_interleave(group, 0)
+    full = torch.nn.functional.scaled_dot_product_attention(qt, kt, vt, is_causal=True)
+    full = full.permute(1, 0, 2).numpy()
+    for R in (1, 5, 22, 23):
+        o = _sdpa(q[T - R:], k, v, suffix_positions(T, R), group)
+        assert np.max(np.abs(o - full[T - R:])) < 1e-12
+
+
 def pin_attention_special(attention):
     """Special cases: a lone visible key returns its value; equal keys give the mean of
     the visible values; one-hot values expose the softmax rows, which are >= 0, zero on

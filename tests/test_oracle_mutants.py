@@ -176,6 +176,21 @@ def test_attention_mutants_caught(name):
     assert (_fails(P.pin_attention_library, m) or _fails(P.pin_attention_special, m))
 
 
+SUFFIX_POSITION_MUTANTS = {
+    # the suffix shifted one past the cache end
+    "start_plus_one": lambda T, R: np.arange(T - R + 1, T + 1, dtype=np.int64),
+    # positions counted from the suffix start instead of the cache start
+    "from_zero": lambda T, R: np.arange(R, dtype=np.int64),
+    # one token short at the end
+    "one_short": lambda T, R: np.arange(T - R, T - 1, dtype=np.int64),
+}
+
+
+@pytest.mark.parametrize("name", sorted(SUFFIX_POSITION_MUTANTS))
+def test_suffix_position_mutants_caught(name):
+    assert _fails(P.pin_suffix_positions, SUFFIX_POSITION_MUTANTS[name])
+
+
 def test_softcap_mutants_caught():
     def cap_before_scale(q, k, v, q_pos, group, softcap=None):
         q = np.asarray(q, float); k = np.asarray(k, float); v = np.asarray(v, float)

@@ -103,3 +103,7 @@ def test_slb_scores():
 
 def test_slb_route():
     P.pin_slb_route(oracle.slb_route)
+
+
+def test_suffix_positions():
+    P.pin_suffix_positions(oracle.suffix_positions)
