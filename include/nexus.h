@@ -155,9 +155,10 @@ int32_t nexus_version(void);
 
 /* Synchronises `stream`, then reports NEXUS_ETIMEOUT if any kernel of this
  * library on the current device gave up a bounded wait since the last call
- * (and clears that record), NEXUS_ERANGE if nexus_suffix_qkv met a page id
- * outside the pool (and skipped that token's cache write), NEXUS_ECUDA if the
- * stream reports an error, else NEXUS_OK. */
+ * (and clears that record), NEXUS_ERANGE if nexus_suffix_qkv or the splice
+ * kernel (nexus_splice_kv, nexus_rope_rerotate, nexus_rope_rerotate_f32) met a
+ * page id outside the pool in a device page table (and skipped the writes that
+ * needed it), NEXUS_ECUDA if the stream reports an error, else NEXUS_OK. */
 nexus_status nexus_device_status(nexus_stream stream);
 
 /* Self-test of the failure path above, for callers that want to see it work on
@@ -306,7 +307,13 @@ nexus_status nexus_plan_splice(nexus_page_pool* pool, const int32_t* h_old_pt,
  *                  id is range-checked and destination rows are checked not
  *                  to overlap each other or any source row (NEXUS_EOVERLAP);
  *                  a segment may read and write the same rows only if it is
- *                  K-only (an in-place rotation).
+ *                  K-only (an in-place rotation). Either way the kernel checks
+ *                  each page id it reads from the device table against the
+ *                  pool before using it: the rows of one destination page
+ *                  whose ids (destination, or a source page) fall outside
+ *                  [0, n_pages) are skipped whole, never dereferenced, and
+ *                  nexus_device_status then reports NEXUS_ERANGE. Overlap is
+ *                  only checked with the host tables.
  *   blocks         host array of n_blocks descriptors; each block's RoPE
  *                  parameters and shape must match the cache
  *                  (NEXUS_EROPE_MISMATCH / NEXUS_ELAYOUT)
@@ -489,11 +496,13 @@ size_t nexus_attention_workspace_size(int32_t n_seqs, const int32_t* h_kv_len,
  * Arguments, results and errors are those of nexus_suffix_attention, without
  * the workspace: the split-KV partials live in a 32 MiB array inside the
  * library, which every GPU that loads the library holds until the process
- * exits. Requests whose partials need more than 32 MiB (see
+ * exits. Arguments are checked first, exactly as nexus_suffix_attention checks
+ * them; then requests whose partials need more than 32 MiB (see
  * nexus_attention_workspace_size) return NEXUS_ENOMEM before any launch; pass
- * split_kv = 1 to need none. The first call on each device looks up the array's
- * device address with that device current; make that first call before any
- * stream capture. Every call shares the one array and overwrites what the
+ * split_kv = 1 to need none. The first call in each CUDA context (the current
+ * device's primary context, unless the caller made another one current) looks
+ * up the array's device address in that context and remembers it; make that
+ * first call before any stream capture. Every call shares the one array and overwrites what the
  * previous call left (nothing in it needs to start at zero), so calls that may
  * run at the same time on the GPU (different streams, no ordering between
  * them) race; order them on one stream or with events. Allocates nothing. */
@@ -528,7 +537,11 @@ nexus_status nexus_suffix_attention_noalloc(const nexus_kv_cache* cache,
  * owns the memory and returns it with nexus_host_free, giving the same size. */
 nexus_status nexus_host_alloc(size_t bytes, void** out);
 /* Unregisters and unmaps memory from nexus_host_alloc. No copy may still be
- * reading or writing it. NULL is a no-op; NEXUS_EINVAL for bytes == 0. */
+ * reading or writing it. NULL is a no-op. NEXUS_EINVAL, with nothing changed,
+ * for bytes == 0, an address nexus_host_alloc did not return (or already
+ * freed), or a size that maps to a different length than that allocation's;
+ * NEXUS_ECUDA if the driver refuses to unregister it (the memory then stays
+ * mapped and may be freed again later). */
 nexus_status nexus_host_free(void* p, size_t bytes);
 
 #ifdef __cplusplus

@@ -98,7 +98,7 @@ __device__ __forceinline__ Work decode_work(const AttnLaunch& p) {
     if (p.tile_prefix[mid] <= rev) lo = mid; else hi = mid - 1;
   }
   w.seq = lo;
-  const int pair = rev - p.tile_prefix[lo];
+  const int pair = rev - p.tile_prefix[lo] + p.pair0[lo];
   w.kv = blockIdx.y;
   w.layer_rel = blockIdx.z / p.splits;
   w.split = blockIdx.z % p.splits;
@@ -163,6 +163,12 @@ __device__ __forceinline__ void mma_bf16_ts(uint32_t d_tmem, uint32_t a_tmem, ui
       "}\n" ::"r"(d_tmem),
       "r"(a_tmem), "l"(b_desc), "r"(idesc), "r"(accumulate)
       : "memory");
+}
+
+__device__ __forceinline__ void tmem_st4(uint32_t taddr, const uint32_t (&r)[4]) {
+  asm volatile("tcgen05.st.sync.aligned.32x32b.x4.b32 [%0], {%1,%2,%3,%4};" ::"r"(taddr),
+               "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3])
+               : "memory");
 }
 
 __device__ __forceinline__ void tmem_st8(uint32_t taddr, const uint32_t (&r)[8]) {
@@ -244,9 +250,25 @@ __device__ __forceinline__ void issue_pv(uint32_t t_o, uint32_t t_s, uint64_t dv
     mma_bf16_ts(t_o, t_s + kk * 8, dv + kk * v_step, idesc, (!first || kk > 0) ? 1u : 0u);
 }
 
+// The first P V product of a tile pair with short rows: O = P V over key tile
+// 0 with P read twice, as bf16 from columns 0..63 and as its bf16 remainder
+// P - bf16(P) from columns 64..127, so O accumulates P at about 16 bits.
+__device__ __forceinline__ void issue_pv_rem(uint32_t t_o, uint32_t t_s, uint64_t dv,
+                                             uint64_t v_step, uint32_t idesc) {
+#pragma unroll
+  for (int kk = 0; kk < BN / 16; ++kk)
+    mma_bf16_ts(t_o, t_s + kk * 8, dv + kk * v_step, idesc, kk > 0 ? 1u : 0u);
+#pragma unroll
+  for (int kk = 0; kk < BN / 16; ++kk)
+    mma_bf16_ts(t_o, t_s + BN / 2 + kk * 8, dv + kk * v_step, idesc, 1u);
+}
+
 // kSoftcap: attention-logit soft-capping (Sec. V-B): the scaled score s becomes
-// cap * tanh(s / cap) before the softmax.
-template <bool kSoftcap>
+// cap * tanh(s / cap) before the softmax. kShort: the launch covers the tile
+// pairs holding rows that see fewer than 128 keys (see short_rows below); the
+// host gives all other pairs to the kShort = false kernel, which carries none of
+// that code (its presence alone slowed the loops of every step by 1-2 %).
+template <bool kSoftcap, bool kShort>
 __global__ void __launch_bounds__(kThreads, 1)
 attention_kernel(const __grid_constant__ AttnLaunch p, const __grid_constant__ AttnMaps maps) {
   extern __shared__ uint8_t smem_raw[];
@@ -267,6 +289,12 @@ attention_kernel(const __grid_constant__ AttnLaunch p, const __grid_constant__ A
   const int layer = p.layer_begin + w.layer_rel;
   const int n_tiles = w.n_tiles;
   const int n_q = w.has_b ? 2 : 1;
+  // Rows that see fewer than 128 keys (positions below 127, all their keys in
+  // the sequence's key tile 0) take P at about 16 bits in that tile: bf16
+  // rounding of a few large weights would otherwise show in O (up to 2^-9 of
+  // |v| per weight). Only a CTA starting at key tile 0 whose first row lies
+  // there has such rows; every other CTA runs exactly the plain bf16 path.
+  const bool short_rows = kShort && w.kt_begin == 0 && w.pos0[0] < BN - 1;
 
   // ---- setup: zero the Q rows no TMA box writes, init barriers, alloc TMEM
   {
@@ -441,8 +469,18 @@ attention_kernel(const __grid_constant__ AttnLaunch p, const __grid_constant__ A
           if (!ok) break;
           if (lane == 0) {
             tc_fence_after();
-            issue_pv(tmem + TM_O + x * 128, tmem + TM_S + x * 128, st ? dv1 : dv0, v_step,
-                     idesc_pv, j == 0);
+            if constexpr (kShort) {
+              // short rows: key tile 0 also reads the remainder of P
+              if (short_rows && j == 0)
+                issue_pv_rem(tmem + TM_O + x * 128, tmem + TM_S + x * 128, st ? dv1 : dv0,
+                             v_step, idesc_pv);
+              else
+                issue_pv(tmem + TM_O + x * 128, tmem + TM_S + x * 128, st ? dv1 : dv0, v_step,
+                         idesc_pv, j == 0);
+            } else {
+              issue_pv(tmem + TM_O + x * 128, tmem + TM_S + x * 128, st ? dv1 : dv0, v_step,
+                       idesc_pv, j == 0);
+            }
             if (x == n_q - 1) mma_commit(bar(B_VE + st));
             if (more) {
               issue_s(tmem + TM_S + x * 128, x ? dq1 : dq0, nst ? dk1 : dk0, idesc_qk,
@@ -554,6 +592,33 @@ attention_kernel(const __grid_constant__ AttnLaunch p, const __grid_constant__ A
           tmem_st8(t_s + q * 8, pk);   // P over the first 64 columns of S
         }
       };
+      // The same pass for short rows' key tile 0, which also writes the bf16
+      // remainder P - bf16(P) over columns 64..127, four columns of each at a
+      // time (the score row already holds 128 of the thread's registers).
+      auto pass_rem = [&](float neg_m) {
+        const float2 sc2 = make_float2(sc, sc);
+        const float2 nm2 = make_float2(neg_m, neg_m);
+#pragma unroll
+        for (int k = 0; k < 4; ++k) sum[k] = make_float2(0.f, 0.f);
+#pragma unroll
+        for (int q = 0; q < 16; ++q) {
+          uint32_t pk[4], pl[4];
+#pragma unroll
+          for (int e = 0; e < 8; e += 2) {
+            const int c = q * 8 + e;
+            float2 ab = ffma2(make_float2(s[c], s[c + 1]), sc2, nm2);
+            ab.x = ex2_approx(ab.x);
+            ab.y = ex2_approx(ab.y);
+            sum[(e >> 1) & 3] = fadd2(sum[(e >> 1) & 3], ab);
+            pk[e / 2] = pack_bf16x2(ab.x, ab.y);
+            // exact differences: bf16(p) keeps p's leading 8 bits
+            pl[e / 2] = pack_bf16x2(ab.x - __uint_as_float(pk[e / 2] << 16),
+                                    ab.y - __uint_as_float(pk[e / 2] & 0xFFFF0000u));
+          }
+          tmem_st4(t_s + q * 4, pk);
+          tmem_st4(t_s + BN / 2 + q * 4, pl);
+        }
+      };
       auto row_max = [&]() -> float {
         return fmaxf(fmax3(mxa[0], mxa[1], mxa[2]),
                      fmaxf(fmax3(mxa[3], mxa[4], mxa[5]), fmaxf(mxa[6], mxa[7])));
@@ -570,7 +635,7 @@ attention_kernel(const __grid_constant__ AttnLaunch p, const __grid_constant__ A
       const bool have_max = __all_sync(0xffffffffu, m_run != -INFINITY);
       bool check = true;
       if (have_max) {
-        pass(-m_run);
+        pass(-m_run);   // never short rows' key tile 0: no running max yet there
         const float rowsum = ((sum[0].x + sum[0].y) + (sum[1].x + sum[1].y)) +
                              ((sum[2].x + sum[2].y) + (sum[3].x + sum[3].y));
         check = !(rowsum < 256.f);
@@ -591,7 +656,12 @@ attention_kernel(const __grid_constant__ AttnLaunch p, const __grid_constant__ A
           if (m_run != -INFINITY) { alpha = ex2_approx(m_run - mxs); rescale = true; }
           m_run = mxs;
         }
-        pass(m_run == -INFINITY ? 0.f : -m_run);
+        if constexpr (kShort) {
+          if (short_rows && j == 0) pass_rem(m_run == -INFINITY ? 0.f : -m_run);
+          else pass(m_run == -INFINITY ? 0.f : -m_run);
+        } else {
+          pass(m_run == -INFINITY ? 0.f : -m_run);
+        }
         if (__any_sync(0xffffffffu, rescale)) {
           // PV_x(j-1) is complete: this step's S-full barrier was committed after it.
 #pragma unroll 1
@@ -738,7 +808,9 @@ cudaError_t launch_wait_selftest(uint64_t budget_ns, cudaStream_t stream) {
 cudaError_t launch_attention(const AttnLaunch& p, const AttnMaps& maps, cudaStream_t stream) {
   if (p.total_tiles <= 0 || p.n_layers_call <= 0) return cudaSuccess;
   static_assert(kSmemBytes <= 227 * 1024, "shared memory budget");
-  auto kernel = p.softcap_out > 0.f ? attention_kernel<true> : attention_kernel<false>;
+  auto kernel = p.softcap_out > 0.f
+                    ? (p.short_rows ? attention_kernel<true, true> : attention_kernel<true, false>)
+                    : (p.short_rows ? attention_kernel<false, true> : attention_kernel<false, false>);
   cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        (int)kSmemBytes);
   if (e != cudaSuccess) return e;
@@ -781,26 +853,76 @@ namespace {
 constexpr size_t kStaticScratchBytes = size_t(32) << 20;   // 32 MiB
 static __device__ __align__(256) unsigned char g_static_split_scratch[kStaticScratchBytes];
 
-constexpr int kMaxScratchDevices = 64;
+// A __device__ array's address belongs to the CUDA context that loaded the
+// module, not to the device: after cudaDeviceReset, or under a context a
+// plug-in made current itself, the array may sit elsewhere. The address is
+// therefore remembered per context, keyed by the context's unique id (ids are
+// never reused within a process, unlike context handles).
+using CtxGetCurrentFn = CUresult (*)(CUcontext*);
+using CtxGetIdFn = CUresult (*)(CUcontext, unsigned long long*);
+struct ScratchEntry {
+  unsigned long long ctx_id;
+  void* addr;
+};
+constexpr int kMaxScratchContexts = 64;
 std::mutex g_scratch_mu;
-void* g_scratch_addr[kMaxScratchDevices] = {};
+ScratchEntry g_scratch[kMaxScratchContexts] = {};
+int g_scratch_n = 0, g_scratch_next = 0;
 
-// Device address of the array on the current device. Host code cannot use the
-// array's name as a device pointer, so the address is looked up once per
-// device (with that device current) and remembered.
-cudaError_t static_scratch_address(void** out) {
-  int dev = 0;
-  cudaError_t e = cudaGetDevice(&dev);
-  if (e != cudaSuccess) return e;
-  if (dev < 0 || dev >= kMaxScratchDevices) return cudaErrorInvalidDevice;
-  std::lock_guard<std::mutex> lock(g_scratch_mu);
-  if (!g_scratch_addr[dev]) {
-    void* p = nullptr;
-    e = cudaGetSymbolAddress(&p, g_static_split_scratch);
-    if (e != cudaSuccess) return e;
-    g_scratch_addr[dev] = p;
+template <typename Fn>
+Fn driver_entry(const char* name) {
+  void* f = nullptr;
+  cudaDriverEntryPointQueryResult q;
+  if (cudaGetDriverEntryPointByVersion(name, &f, 12000, cudaEnableDefault, &q) != cudaSuccess ||
+      q != cudaDriverEntryPointSuccess) {
+    cudaGetLastError();
+    return nullptr;
   }
-  *out = g_scratch_addr[dev];
+  return reinterpret_cast<Fn>(f);
+}
+
+// Unique id of the current context; false if none is current or the driver
+// cannot tell.
+bool current_context_id(unsigned long long* id) {
+  static CtxGetCurrentFn get_current = nullptr;
+  static CtxGetIdFn get_id = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    get_current = driver_entry<CtxGetCurrentFn>("cuCtxGetCurrent");
+    get_id = driver_entry<CtxGetIdFn>("cuCtxGetId");
+  });
+  if (!get_current || !get_id) return false;
+  CUcontext ctx = nullptr;
+  if (get_current(&ctx) != CUDA_SUCCESS || !ctx) return false;
+  return get_id(ctx, id) == CUDA_SUCCESS;
+}
+
+// Device address of the array in the current context. Host code cannot use the
+// array's name as a device pointer, so the address is looked up once per
+// context (cudaGetSymbolAddress, with that context current) and remembered.
+cudaError_t static_scratch_address(void** out) {
+  std::lock_guard<std::mutex> lock(g_scratch_mu);
+  unsigned long long id = 0;
+  if (current_context_id(&id)) {
+    for (int i = 0; i < g_scratch_n; ++i)
+      if (g_scratch[i].ctx_id == id) {
+        *out = g_scratch[i].addr;
+        return cudaSuccess;
+      }
+  }
+  void* p = nullptr;
+  const cudaError_t e = cudaGetSymbolAddress(&p, g_static_split_scratch);
+  if (e != cudaSuccess) return e;
+  // The lookup may have made the runtime's primary context current.
+  if (current_context_id(&id)) {
+    ScratchEntry& slot = g_scratch_n < kMaxScratchContexts ? g_scratch[g_scratch_n++]
+                                                           : g_scratch[g_scratch_next];
+    if (g_scratch_n == kMaxScratchContexts)
+      g_scratch_next = (g_scratch_next + 1) % kMaxScratchContexts;
+    slot.ctx_id = id;
+    slot.addr = p;
+  }
+  *out = p;
   return cudaSuccess;
 }
 }  // namespace
@@ -811,11 +933,8 @@ extern "C" nexus_status nexus_suffix_attention_noalloc(
     int32_t n_seqs, const int32_t* h_rows, const int32_t* h_kv_len, const int32_t* h_q_len,
     const void* q, void* out, float* lse, int32_t n_q_heads, int32_t layer_begin,
     int32_t layer_end, int32_t split_kv, nexus_stream stream) {
-  if (!cache) return NEXUS_EINVAL;
-  const size_t need = nexus_attention_workspace_size(n_seqs, h_kv_len, h_q_len, n_q_heads,
-                                                     cache->n_kv_heads, layer_end - layer_begin,
-                                                     split_kv, nullptr);
-  if (need > nexus::kStaticScratchBytes) return NEXUS_ENOMEM;
+  // Arguments are validated by nexus_suffix_attention, which also returns
+  // NEXUS_ENOMEM (before any launch) when the partials need more than the array.
   void* scratch = nullptr;
   if (nexus::static_scratch_address(&scratch) != cudaSuccess) {
     cudaGetLastError();

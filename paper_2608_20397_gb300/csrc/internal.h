@@ -54,6 +54,8 @@ struct SpliceLaunch {
 };
 
 cudaError_t launch_splice(const SpliceLaunch& p, cudaStream_t stream);
+// Reads and clears the splice kernel's record of a page id outside the pool.
+cudaError_t splice_take_status(unsigned int* bad_page, cudaStream_t stream);
 
 // -------------------------------------------------------------- page copy
 constexpr int kMaxPageCopies = 2048;
@@ -105,6 +107,8 @@ struct AttnLaunch {
   float softcap_out;        // soft-capping: cap log2(e); 0 = no soft-capping
   int32_t tile_prefix[kMaxSeqs + 1];   // first CTA (tile pair) of each sequence
   AttnSeq seq[kMaxSeqs];
+  int32_t pair0[kMaxSeqs];  // first tile pair of each sequence in this launch
+  int32_t short_rows;       // this launch's tile pairs hold rows that see fewer than 128 keys
 };
 
 struct AttnMaps {

@@ -11,6 +11,7 @@
 #include <cmath>
 #include <cstdio>
 #include <cstring>
+#include <map>
 #include <memory>
 #include <mutex>
 #include <vector>
@@ -302,36 +303,52 @@ nexus_status plan_attention(int32_t n_seqs, const int32_t* kv_len, const int32_t
   const int32_t tile_tokens = 128 / group;
   AttnPlan pl;
   int64_t tok = 0, tiles = 0;
+  double key_tiles = 0.0;   // key tiles over all CTAs of one KV head (no split)
   for (int32_t s = 0; s < n_seqs; ++s) {
     if (q_len[s] < 0 || kv_len[s] < q_len[s]) return NEXUS_EINVAL;
     tok += q_len[s];
-    tiles += ((q_len[s] + tile_tokens - 1) / tile_tokens + 1) / 2;   // CTAs: pairs of query tiles
+    const int32_t q_tiles = (q_len[s] + tile_tokens - 1) / tile_tokens;
+    const int32_t pairs = (q_tiles + 1) / 2;   // CTAs: pairs of query tiles
+    tiles += pairs;
     if (q_len[s] > 0) pl.kt_max = std::max(pl.kt_max, (kv_len[s] + 127) / 128);
+    for (int32_t k = 0; k < pairs; ++k) {
+      const int64_t last_tok = std::min<int64_t>(q_len[s], (2 * k + 2) * int64_t{tile_tokens}) - 1;
+      key_tiles += static_cast<double>((kv_len[s] - q_len[s] + last_tok) / 128 + 1);
+    }
   }
   if (tok > 0x7FFFFFFF || tiles > 0x7FFFFFFF) return NEXUS_ERANGE;
   pl.n_tok = static_cast<int32_t>(tok);
   pl.total_tiles = static_cast<int32_t>(tiles);
   if (split_kv < 0) return NEXUS_EINVAL;
   if (split_kv == 0) {
-    // Balance waves of one-CTA-per-SM work against the per-split merge. A CTA
-    // also pays a fixed start (Q and the first K/V tiles, filling the pipeline)
-    // and end (its partial rows): about four key tiles' worth, measured on the
-    // c5 suffix (64 queries over 34816 keys: 9 splits in one wave 72 us a
-    // layer, 19 splits in two waves 84 us).
-    constexpr double kCtaFixedTiles = 4.0;
+    // Waves of one-CTA-per-SM work against the merge of the partials, in units
+    // of one key-tile step of a CTA (~1.66 us). A CTA runs its share of the mean
+    // key tiles per CTA plus a fixed start (Q and the first K/V tiles, filling
+    // the pipeline) and end (its partial rows) worth about four steps; the merge
+    // reads every split's partial rows (~3 us plus 4 MB/us). Calibrated on the
+    // c5 suffix (9 splits in one wave, 72 us a layer) and on sweeps of c2 and
+    // c3, whose best counts this model picks; a split is taken only where it is
+    // predicted to save at least 10 %.
+    constexpr double kCtaFixedSteps = 4.0, kStepUs = 1.66, kMergeBytesPerUs = 4.0e6;
     const int64_t ctas = tiles * n_kv_heads * std::max(1, n_layers_call);
     const int sms = num_sms();
+    const double rows = static_cast<double>(tok) * n_q_heads * std::max(1, n_layers_call);
+    const double mean_tiles = tiles > 0 ? key_tiles / static_cast<double>(tiles) : 0.0;
+    auto cost = [&](int s) {
+      const double waves = std::ceil(static_cast<double>(ctas) * s / sms);
+      double c = waves * (mean_tiles / s + kCtaFixedSteps);
+      if (s > 1) c += (3.0 + s * rows * (kHeadDim * 4 + 4) / kMergeBytesPerUs) / kStepUs;
+      return c;
+    };
     int best = 1;
-    double best_cost = 1e300;
-    // Splitting the keys only pays when the query tiles alone fill less than
-    // one wave of the GPU (short suffixes over deep caches).
-    if (ctas > 0 && ctas < sms && pl.kt_max > 0) {
-      for (int s = 1; s <= std::min<int>(kMaxSplits, pl.kt_max); ++s) {
-        const double waves = std::ceil(static_cast<double>(ctas) * s / sms);
-        const double cost = waves * (std::ceil(static_cast<double>(pl.kt_max) / s) + kCtaFixedTiles) +
-                            (s > 1 ? 2.0 : 0.0);
-        if (cost < best_cost - 1e-9) { best_cost = cost; best = s; }
+    if (ctas > 0 && pl.kt_max > 1) {
+      const double c1 = cost(1);
+      double best_cost = c1;
+      for (int s = 2; s <= std::min<int>(kMaxSplits, pl.kt_max); ++s) {
+        const double c = cost(s);
+        if (c < best_cost - 1e-9) { best_cost = c; best = s; }
       }
+      if (best_cost > 0.9 * c1) best = 1;
     }
     pl.splits = best;
   } else {
@@ -404,17 +421,46 @@ nexus_status attention_impl(const nexus_kv_cache* c, const int32_t* d_pt, int32_
     p->part_o = static_cast<float*>(ws);
     p->part_lse = static_cast<float*>(ws) + static_cast<size_t>(pl.splits) * rows * kHeadDim;
   }
-  int32_t tiles = 0, off = 0;
+  // Tile pairs whose first query row sees fewer than 128 keys (position below
+  // 127) go to a launch of their own (the kernel's short-row instantiation);
+  // the rest, usually all but a few pairs, to the plain kernel.
+  const int32_t tt = p->tile_tokens;
+  std::vector<int32_t> short_pairs(static_cast<size_t>(n_seqs), 0);
+  int32_t n_short = 0;
+  int32_t off = 0;
   for (int32_t s = 0; s < n_seqs; ++s) {
-    p->tile_prefix[s] = tiles;
     p->seq[s].kv_len = kv_len[s];
     p->seq[s].q_len = q_len[s];
     p->seq[s].q_off = off;
     p->seq[s].pt_row = h_rows ? h_rows[s] : s;
-    tiles += ((q_len[s] + p->tile_tokens - 1) / p->tile_tokens + 1) / 2;
     off += q_len[s];
+    const int32_t pairs = ((q_len[s] + tt - 1) / tt + 1) / 2;
+    const int32_t c = kv_len[s] - q_len[s];   // position of the sequence's first query
+    if (pairs > 0 && c < 127)
+      short_pairs[s] = std::min(pairs, (127 - c + 2 * tt - 1) / (2 * tt));
+    n_short += short_pairs[s];
+  }
+  std::unique_ptr<AttnLaunch> ps;
+  if (n_short > 0) {
+    ps.reset(new AttnLaunch(*p));
+    ps->short_rows = 1;
+    int32_t t = 0;
+    for (int32_t s = 0; s < n_seqs; ++s) {
+      ps->tile_prefix[s] = t;
+      ps->pair0[s] = 0;
+      t += short_pairs[s];
+    }
+    ps->tile_prefix[n_seqs] = t;
+    ps->total_tiles = t;
+  }
+  int32_t tiles = 0;
+  for (int32_t s = 0; s < n_seqs; ++s) {
+    p->tile_prefix[s] = tiles;
+    p->pair0[s] = short_pairs[s];
+    tiles += ((q_len[s] + tt - 1) / tt + 1) / 2 - short_pairs[s];
   }
   p->tile_prefix[n_seqs] = tiles;
+  p->total_tiles = tiles;
 
   AttnMaps maps;
   const uint64_t tok_stride = static_cast<uint64_t>(n_q_heads) * kHeadDim * 2;
@@ -446,6 +492,7 @@ nexus_status attention_impl(const nexus_kv_cache* c, const int32_t* d_pt, int32_
       return NEXUS_ECUDA;
   }
   if (launch_attention(*p, maps, stream) != cudaSuccess) return NEXUS_ECUDA;
+  if (ps && launch_attention(*ps, maps, stream) != cudaSuccess) return NEXUS_ECUDA;
   if (pl.splits > 1 && launch_attn_combine(*p, stream) != cudaSuccess) return NEXUS_ECUDA;
   return NEXUS_OK;
 }
@@ -455,15 +502,16 @@ nexus_status attention_impl(const nexus_kv_cache* c, const int32_t* d_pt, int32_
 extern "C" {
 
 nexus_status nexus_device_status(nexus_stream stream) {
-  unsigned int flag = 0, qkv_timeout = 0, bad_page = 0, slb_timeout = 0;
+  unsigned int flag = 0, qkv_timeout = 0, bad_page = 0, slb_timeout = 0, splice_bad = 0;
   if (attention_take_timeout(&flag, static_cast<cudaStream_t>(stream)) != cudaSuccess ||
       qkv_take_status(&qkv_timeout, &bad_page, static_cast<cudaStream_t>(stream)) != cudaSuccess ||
-      slb_take_timeout(&slb_timeout, static_cast<cudaStream_t>(stream)) != cudaSuccess) {
+      slb_take_timeout(&slb_timeout, static_cast<cudaStream_t>(stream)) != cudaSuccess ||
+      splice_take_status(&splice_bad, static_cast<cudaStream_t>(stream)) != cudaSuccess) {
     cudaGetLastError();
     return NEXUS_ECUDA;
   }
   if (flag || qkv_timeout || slb_timeout) return NEXUS_ETIMEOUT;
-  return bad_page ? NEXUS_ERANGE : NEXUS_OK;
+  return (bad_page || splice_bad) ? NEXUS_ERANGE : NEXUS_OK;
 }
 
 nexus_status nexus_selftest_wait(uint32_t budget_us, nexus_stream stream) {
@@ -833,6 +881,14 @@ static size_t host_huge_page() {
   return hp;
 }
 
+// Mappings handed out by nexus_host_alloc (address -> length), so that
+// nexus_host_free unmaps only what this library mapped, at the length it mapped.
+static std::mutex g_host_maps_mu;
+static std::map<void*, size_t>& host_maps() {
+  static std::map<void*, size_t> m;
+  return m;
+}
+
 static size_t host_mapping_len(size_t bytes, size_t* align) {
   const size_t hp = host_huge_page();
   const size_t unit = (hp && bytes >= hp / 4) ? hp : host_base_page();
@@ -876,6 +932,10 @@ nexus_status nexus_host_alloc(size_t bytes, void** out) {
     munmap(p, len);
     return NEXUS_ECUDA;
   }
+  {
+    std::lock_guard<std::mutex> lock(g_host_maps_mu);
+    host_maps()[p] = len;
+  }
   *out = p;
   return NEXUS_OK;
 }
@@ -885,10 +945,18 @@ nexus_status nexus_host_free(void* p, size_t bytes) {
   if (bytes == 0) return NEXUS_EINVAL;
   size_t align = 0;
   const size_t len = host_mapping_len(bytes, &align);
-  const bool unregistered = cudaHostUnregister(p) == cudaSuccess;
-  if (!unregistered) cudaGetLastError();
+  std::lock_guard<std::mutex> lock(g_host_maps_mu);
+  auto it = host_maps().find(p);
+  if (it == host_maps().end() || it->second != len) return NEXUS_EINVAL;
+  if (cudaHostUnregister(p) != cudaSuccess) {
+    // Still registered: leave it mapped (and recorded) rather than unmap pages
+    // the driver may still reach.
+    cudaGetLastError();
+    return NEXUS_ECUDA;
+  }
   munmap(p, len);
-  return unregistered ? NEXUS_OK : NEXUS_ECUDA;
+  host_maps().erase(it);
+  return NEXUS_OK;
 }
 
 size_t nexus_attention_workspace_size(int32_t n_seqs, const int32_t* h_kv_len,

@@ -13,6 +13,11 @@
 #include "internal.h"
 
 namespace nexus {
+
+// Set when a page id read from a device page table lies outside the pool; the
+// piece that met it is skipped whole (nothing read or written through it).
+__device__ unsigned int g_splice_bad_page = 0;
+
 namespace {
 
 constexpr int kThreads = 256;
@@ -127,6 +132,23 @@ __global__ void __launch_bounds__(kThreads) splice_kernel(const __grid_constant_
   if (ns <= 0) return;
   const int slot0 = (sg.dst_start + r0) % kPageSize;
   const int32_t dpage = p.page_tables[(int64_t)sg.dst_row * p.max_pages + dpage_idx];
+  // Every page id this piece goes through (its destination page and, for a
+  // cache source, the at most two pages its source rows span) is checked
+  // against the pool before any access: the device table may hold ids the host
+  // never saw. A bad id skips the piece and is recorded for nexus_device_status.
+  {
+    bool bad = dpage < 0 || dpage >= p.n_pages;
+    if (sg.src_k == nullptr) {
+      const int64_t srow = (int64_t)sg.src_row * p.max_pages;
+      const int32_t sp0 = p.page_tables[srow + (sg.src_start + r0) / kPageSize];
+      const int32_t sp1 = p.page_tables[srow + (sg.src_start + r1 - 1) / kPageSize];
+      bad = bad || sp0 < 0 || sp0 >= p.n_pages || sp1 < 0 || sp1 >= p.n_pages;
+    }
+    if (bad) {
+      if (threadIdx.x == 0) atomicOr(&g_splice_bad_page, 1u);
+      return;
+    }
+  }
 
   const bool rotate = sg.delta != 0;
   if (rotate && threadIdx.x < kHeadDim / 2) {
@@ -438,6 +460,15 @@ cudaError_t launch_splice(const SpliceLaunch& p, cudaStream_t stream) {
   }
   splice_kernel<<<(unsigned)blocks, kThreads, smem, stream>>>(p);
   return cudaGetLastError();
+}
+
+cudaError_t splice_take_status(unsigned int* bad_page, cudaStream_t stream) {
+  cudaError_t e = cudaStreamSynchronize(stream);
+  if (e != cudaSuccess) return e;
+  e = cudaMemcpyFromSymbol(bad_page, g_splice_bad_page, sizeof(unsigned int));
+  if (e != cudaSuccess) return e;
+  const unsigned int zero = 0;
+  return cudaMemcpyToSymbol(g_splice_bad_page, &zero, sizeof(unsigned int));
 }
 
 cudaError_t launch_page_copy(const PageCopyLaunch& p, cudaStream_t stream) {

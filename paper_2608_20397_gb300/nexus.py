@@ -557,6 +557,7 @@ class _HostMapping:
     is gone."""
 
     def __init__(self, nbytes: int):
+        self.ptr, self.nbytes = 0, int(nbytes)   # set before the call that can fail
         p = c_void_p()
         _check("nexus_host_alloc", lib().nexus_host_alloc(int(nbytes), ctypes.byref(p)))
         self.ptr, self.nbytes = int(p.value), int(nbytes)

@@ -6,9 +6,11 @@ Tolerances (written here once, used by every GPU test):
 * re-rotated K (bf16 store): |K - K_oracle| <= 2e-3 + half a bf16 ulp of
   |K_oracle| (the bf16 store alone errs by up to half an ulp, 3.9e-3 at
   |k| in [1, 2)); the float32 output of the same arithmetic: <= 2e-3;
-* attention output (bf16 store): |O - O_oracle| <= 1e-2 + half a bf16 ulp of
-  |O_oracle| (the store alone errs by up to half an ulp, 1.6e-2 at |o| in
-  [4, 8)) and relative L2 <= 5e-3; LSE max abs <= 1e-2.
+* attention output: |O - O_oracle| <= 1e-2 wherever the bf16 output can hold a
+  value that close (|O_oracle| < 4, where half a bf16 ulp is at most 7.8e-3);
+  from |O_oracle| >= 4 on, half an ulp alone is 1.6e-2 or more, so there the
+  bound is 1e-2 plus half a bf16 ulp of |O_oracle|; relative L2 <= 5e-3; LSE
+  max abs <= 1e-2.
 """
 from __future__ import annotations
 
@@ -39,10 +41,15 @@ def assert_k_close(got: np.ndarray, want: np.ndarray, what=""):
     assert not bad.any(), f"{what}: {bad.sum()} K elements out of tolerance, worst {err.max():.3e}"
 
 
+def attn_abs_bound(want: np.ndarray) -> np.ndarray:
+    """1e-2, widened by half a bf16 ulp only where that half ulp is itself 1.6e-2 or more."""
+    return np.where(np.abs(want) < 4.0, ATTN_ABS, ATTN_ABS + half_ulp_bf16(want))
+
+
 def assert_attn_close(got: np.ndarray, want: np.ndarray, got_lse=None, want_lse=None, what=""):
     err = np.abs(got - want)
     rel = np.linalg.norm(got - want) / max(np.linalg.norm(want), 1e-30)
-    bad = err > ATTN_ABS + half_ulp_bf16(want)
+    bad = err > attn_abs_bound(want)
     assert not bad.any(), f"{what}: {bad.sum()} outputs out of tolerance, max abs {err.max():.3e}"
     assert rel <= ATTN_REL, f"{what}: rel L2 {rel:.3e}"
     if got_lse is not None:

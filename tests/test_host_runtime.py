@@ -428,6 +428,11 @@ def test_host_staging_argument_checks():
     assert L.nexus_host_alloc(4096, None) == nexus.EINVAL
     assert L.nexus_host_alloc(1 << 60, ctypes.byref(out)) == nexus.EINVAL
     assert L.nexus_host_free(None, 4096) == nexus.OK
+    # memory the library did not map is refused before anything is unmapped
+    buf = ctypes.create_string_buffer(1 << 16)
+    assert L.nexus_host_free(ctypes.c_void_p(ctypes.addressof(buf)), 1 << 16) == nexus.EINVAL
+    assert L.nexus_host_free(ctypes.c_void_p(ctypes.addressof(buf)), 0) == nexus.EINVAL
+    buf[0] = b"x"                                   # still mapped and writable
     import torch
     if not torch.cuda.is_available():
         # no driver to register with: nothing is left mapped and NULL comes back

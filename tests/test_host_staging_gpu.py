@@ -41,7 +41,12 @@ def test_direct_alloc_and_free(dev):
     assert L.nexus_host_alloc(5000, ctypes.byref(p)) == nexus.OK and p.value
     assert p.value % 4096 == 0
     ctypes.memset(p.value, 7, 5000)
+    # a size that maps to another length, or an address inside the mapping, is refused
+    assert L.nexus_host_free(p, 1 << 30) == nexus.EINVAL
+    assert L.nexus_host_free(ctypes.c_void_p(p.value + 4096), 100) == nexus.EINVAL
+    assert ctypes.string_at(p.value, 1) == b"\x07"   # still mapped
     assert L.nexus_host_free(p, 5000) == nexus.OK
+    assert L.nexus_host_free(p, 5000) == nexus.EINVAL   # already returned
 
 
 def test_views_keep_the_mapping(dev):

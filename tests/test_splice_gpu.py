@@ -227,3 +227,45 @@ def test_splice_edge_shapes():
         assert nexus.device_status() == nexus.OK
         for si in range(3):
             _check_session(case, si, [0, 1])
+
+
+def test_splice_bad_device_page_is_skipped_and_reported():
+    # Without the host tables the kernel checks the page ids itself: a piece
+    # whose destination or source page lies outside the pool is skipped whole
+    # (nothing read or written through the bad id) and the call reports it.
+    w = workload("c1")                     # 128-row block at depth 300 of 512 (tail 212)
+    clean = SplicedCase(w, DEV)
+    clean.splice()
+    assert nexus.device_status() == nexus.OK
+    want_k, want_v = clean.kp.clone(), clean.vp.clone()
+
+    # destination: page index 20 of the new table (block rows 20..35, positions 320..335)
+    case = SplicedCase(w, DEV)
+    k0, v0 = case.kp.clone(), case.vp.clone()
+    bad = case.h_pt.copy()
+    real = int(bad[1, 20])
+    bad[1, 20] = case.n_pages + 5
+    case.d_pt = torch.as_tensor(bad, device=DEV)
+    case.splice(validate=False)
+    assert nexus.device_status() == nexus.ERANGE
+    assert nexus.device_status() == nexus.OK                 # the record is cleared
+    others = torch.ones(case.n_pages, dtype=torch.bool, device=DEV)
+    others[real] = False
+    for got, want, before in ((case.kp, want_k, k0), (case.vp, want_v, v0)):
+        assert torch.equal(got[:, others].view(torch.int16), want[:, others].view(torch.int16))
+        assert torch.equal(got[:, real].view(torch.int16), before[:, real].view(torch.int16))
+
+    # source: page index 25 of the old table (displaced rows at positions 400..415)
+    case = SplicedCase(w, DEV)
+    k0, v0 = case.kp.clone(), case.vp.clone()
+    bad = case.h_pt.copy()
+    bad[0, 25] = -1
+    case.d_pt = torch.as_tensor(bad, device=DEV)
+    case.splice(validate=False)
+    assert nexus.device_status() == nexus.ERANGE
+    for got, want, before in ((case.kp, want_k, k0), (case.vp, want_v, v0)):
+        g, a, b = (x.view(torch.int16) for x in (got, want, before))
+        # every 16-byte-wide row slice is either the clean result or untouched
+        same = (g == a).all(-1) | (g == b).all(-1)
+        assert bool(same.all())
+        assert not torch.equal(g, a)                       # and something was skipped
