@@ -308,6 +308,8 @@ def main():
                     help="skip the separate timing of the L0 warm arena")
     ap.add_argument("--no-slb", action="store_true",
                     help="skip the separate timing of the INT8 tool scan")
+    ap.add_argument("--no-configs", action="store_true",
+                    help="skip the separate timings of the workloads c1 .. c4")
     ap.add_argument("--layers", type=int, default=48, help="layers of the workload (48 = c5)")
     ap.add_argument("--profile", choices=["reprefill", "reprefill-softcap", "splice", "suffix",
                                           "qkv", "slb"],
@@ -430,6 +432,11 @@ def main():
         slb = _slb_measure(wl, stream, peaks, peak_kind,
                            with_oracle=rank == 0 and world == 1 and not args.no_cpu_baseline)
 
+    configs = None
+    if not args.no_configs:
+        configs = _configs_measure(dev, stream, peaks, peak_kind,
+                                   with_oracle=rank == 0 and world == 1 and not args.no_cpu_baseline)
+
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         f64 = lambda t: t.float().cpu().double().numpy()
@@ -455,6 +462,7 @@ def main():
             "suffix_ms": suf_ms, "suffix_tflops": suf_tflops, "roofline_suffix": roofline_suffix,
             "roofline": roofline, "roofline_splice": roofline_splice,
             "e2e": e2e, "cpu_baseline": cpu, "clocks": clocks, "qkv_recompute": qkv, "l0_arena": arena, "slb_route": slb,
+            "configs": configs,
             "gpu_launches": wl.launches_per_step * args.steps,
         }
         print(json.dumps(line), flush=True)
@@ -884,6 +892,209 @@ def _slb_measure(wl, stream, peaks, peak_kind, with_oracle, reps=200):
         out["cpu_baseline"] = {"value": dt * 1e6, "unit": "us per query", "cores": 1,
                                "kind": "oracle",
                                "sample": "NumPy oracle: one query against 250 x 768 codes"}
+    return out
+
+
+# ---------------------------------------------------- configs c1 .. c4
+class ConfigCase:
+    """One of the workloads c1 .. c4 resident on the device: every session's live
+    rows in a paged pool (N(0, 1) bf16, pages handed out in the workload's
+    order), its compiled blocks, the planned splice (page-table rows 2 s / 2 s + 1
+    before / after the splice) and the suffix queries of each redecode fraction."""
+
+    def __init__(self, name, dev):
+        import torch
+
+        from paper_2608_20397_gb300 import nexus
+        from paper_2608_20397_gb300.workloads import page_order, randn_bf16, workload
+
+        self.torch, self.nexus = torch, nexus
+        w = workload(name)
+        self.w, self.name, self.L, self.vt = w, name, w.n_layers, w.v_transposed
+        S = len(w.sessions)
+        self.kv = [w.spliced_len(s) for s in w.sessions]
+        pages = sum(-(-s.n_past // PAGE) + -(-t // PAGE) + 1 for s, t in zip(w.sessions, self.kv))
+        self.n_pages = pages + 64
+        self.max_pages = max(-(-t // PAGE) for t in self.kv) + 1
+        self.pool = nexus.PagePool(self.n_pages, page_order(self.n_pages, w.seed, w.shuffle_pages))
+        g = torch.Generator(device=dev)
+        g.manual_seed(9000 + w.seed)
+        # Every slot of the pool holds N(0, 1) bf16: the live rows are whatever
+        # the pages hold (the timing does not depend on which values they are).
+        self.kp = torch.empty((self.L, self.n_pages, HKV, PAGE, D), dtype=torch.bfloat16, device=dev)
+        vshape = (self.L, self.n_pages, HKV, D, PAGE) if self.vt else self.kp.shape
+        self.vp = torch.empty(vshape, dtype=torch.bfloat16, device=dev)
+        for l in range(self.L):
+            self.kp[l].normal_(generator=g)
+            self.vp[l].normal_(generator=g)
+        self.cache = nexus.kv_cache(self.kp, self.vp, self.n_pages, self.L, HKV, self.vt,
+                                    rope_theta=w.rope_theta)
+        h_pt = np.full((2 * S, self.max_pages), -1, np.int32)
+        self.blocks, self.segs, self._blk = [], [], []
+        for si, s in enumerate(w.sessions):
+            npg = -(-s.n_past // PAGE)
+            h_pt[2 * si, :npg] = self.pool.alloc(npg)
+            base = len(self.blocks)
+            for j, ins in enumerate(s.inserts):
+                bk = randn_bf16((self.L, ins.length, HKV, D), 20000 + 10 * si + 2 * j, dev)
+                bv = randn_bf16((self.L, ins.length, HKV, D), 20001 + 10 * si + 2 * j, dev)
+                self._blk += [bk, bv]
+                self.blocks.append(nexus.block(bk, bv, ins.length, ins.base_pos, self.L, HKV,
+                                               rope_theta=w.rope_theta))
+            new_pt, segs, _ = nexus.plan_splice(
+                self.pool, h_pt[2 * si], s.n_past, self.max_pages, self.blocks,
+                [(ins.depth, base + j) for j, ins in enumerate(s.inserts)], 2 * si, 2 * si + 1,
+                seg_capacity=4 * len(s.inserts) + 4)
+            h_pt[2 * si + 1] = new_pt
+            self.segs += segs
+        self.h_pt = h_pt
+        self.d_pt = torch.as_tensor(h_pt, device=dev)
+        self.n_rows = 2 * S
+        # every segment moves its rows' K and V: 8192 bytes per row and layer
+        self.moved_rows = sum(int(sg.n_tokens) for sg in self.segs)
+        self.splice_bytes = 8192.0 * self.moved_rows * self.L
+        pcts = w.suffix_pcts or (w.sessions[0].suffix_pct,)
+        self.q_len = {p: [nexus.suffix_len(s.suffix_span, p) for s in w.sessions] for p in pcts}
+
+    def splice(self, stream):
+        self.nexus.splice_kv(self.cache, self.d_pt, None, self.n_rows, self.max_pages, self.blocks,
+                             self.segs, 0, self.L, stream)
+
+    def flops(self, pct):
+        return sum(attn_flops(T, R, self.L) for T, R in zip(self.kv, self.q_len[pct]))
+
+
+def _time_back_to_back(fn, stream, warmup, reps):
+    """Mean CUDA-event time (ms) of `reps` back-to-back calls, enqueued behind a
+    fixed-length sleep so that short launches are timed without host gaps."""
+    import torch
+    for _ in range(warmup):
+        fn()
+    torch.cuda.synchronize()
+    a = torch.cuda.Event(enable_timing=True)
+    b = torch.cuda.Event(enable_timing=True)
+    torch.cuda._sleep(4_000_000)
+    a.record(stream)
+    for _ in range(reps):
+        fn()
+    b.record(stream)
+    torch.cuda.synchronize()
+    return a.elapsed_time(b) / reps
+
+
+def _oracle_config_sample(T, R, budget_s=1.0):
+    """The fp64 oracle on a bounded sample of a config's suffix attention (one
+    layer, rows from the deep end of the suffix, N(0, 1) inputs) and of its
+    splice (a 64-row block into a 64-row cache, one layer). Returns (attention
+    TFLOP/s, splice GB/s, description)."""
+    import oracle
+    from paper_2608_20397_gb300.workloads import randn_bf16
+    f64 = lambda t: t.float().double().numpy()
+    rows_max = min(R, 64)
+    q = f64(randn_bf16((rows_max, HQ, D), 31, "cpu"))
+    k = f64(randn_bf16((T, HKV, D), 32, "cpu"))
+    v = f64(randn_bf16((T, HKV, D), 33, "cpu"))
+    flops, spent, done = 0.0, 0.0, 0
+    while done < rows_max and (spent < budget_s or done == 0):
+        r = min(4, rows_max - done)
+        pos = np.arange(T - done - r, T - done)
+        t0 = time.perf_counter()
+        oracle.attention(q[done:done + r], k, v, pos, HQ // HKV)
+        spent += time.perf_counter() - t0
+        flops += sum(4.0 * D * HQ * (p + 1) for p in pos)
+        done += r
+    live = f64(randn_bf16((1, 64, HKV, D), 34, "cpu"))
+    blk = f64(randn_bf16((1, 64, HKV, D), 35, "cpu"))
+    t0 = time.perf_counter()
+    oracle.splice_sequence(live, live, [(32, blk, blk, 0)])
+    t_spl = time.perf_counter() - t0
+    desc = (f"fp64 NumPy oracle: {done} suffix rows x {HQ} heads over up to {T} keys (one layer), "
+            f"and a 64-row block splice into a 64-row cache (one layer)")
+    return flops / spent / 1e12, 8192.0 * 96 / t_spl / 1e9, desc
+
+
+def _configs_measure(dev, stream, peaks, peak_kind, with_oracle, warmup=3, reps=10):
+    """c1 .. c4 timed one after another, apart from the c5 step: the splice of
+    each (hot, and for the single-layer c1 / c2, whose moved rows fit in L2,
+    also with a 512 MB scratch write between launches) and its suffix attention
+    at every redecode fraction the config names (one launch per layer), each
+    against its roofline, with the fp64 oracle on a bounded sample beside it."""
+    import torch
+    nexus = None
+    peak_tc = peaks["bf16_tflops"]
+    out = {}
+    for name in ("c1", "c2", "c3", "c4"):
+        case = ConfigCase(name, dev)
+        nexus = case.nexus
+        w = case.w
+        line = {"layers": case.L, "sessions": len(w.sessions),
+                "v_layout": "token-innermost" if case.vt else "row-major",
+                "pages": "shuffled" if w.shuffle_pages else "in order",
+                "kv_len": case.kv if len(case.kv) <= 2 else
+                {"min": min(case.kv), "max": max(case.kv), "sum": sum(case.kv)}}
+        ms = _time_back_to_back(lambda: case.splice(stream), stream, warmup, reps)
+        gbs = case.splice_bytes / (ms * 1e-3) / 1e9
+        spl = {"moved_rows_per_layer": case.moved_rows, "bytes": case.splice_bytes,
+               "ms": ms, "gbs": gbs, "frac": gbs / peaks["hbm_gbs"],
+               "bound": "hbm", "peak": peaks["hbm_gbs"], "peak_kind": f"copy, {peak_kind}",
+               "timing": "back to back (moved rows L2-resident where they fit)"}
+        if case.L == 1:
+            flush = torch.empty(512 << 20, dtype=torch.uint8, device=dev)
+            evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+                   for _ in range(reps)]
+            for i in range(warmup + reps):
+                flush.fill_(i & 255)
+                if i >= warmup:
+                    evs[i - warmup][0].record(stream)
+                case.splice(stream)
+                if i >= warmup:
+                    evs[i - warmup][1].record(stream)
+            torch.cuda.synchronize()
+            msf = statistics.mean(a.elapsed_time(b) for a, b in evs)
+            gf = case.splice_bytes / (msf * 1e-3) / 1e9
+            spl.update({"ms_l2_flushed": msf, "gbs_l2_flushed": gf,
+                        "frac_l2_flushed": gf / peaks["hbm_gbs"],
+                        "flush": "512 MB scratch write before each timed launch (events per launch)"})
+            del flush
+        line["splice"] = spl
+        case.splice(stream)
+        torch.cuda.synchronize()
+        sufs = []
+        for pct, ql in case.q_len.items():
+            n_tok = sum(ql)
+            q = torch.empty((case.L, n_tok, HQ, D), dtype=torch.bfloat16, device=dev).normal_()
+            o = torch.empty_like(q)
+            lse = torch.empty((case.L, n_tok, HQ), dtype=torch.float32, device=dev)
+            wsb, splits = nexus.attention_workspace_size(case.kv, ql, HQ, HKV, 1, 0)
+            ws = torch.empty(max(16, wsb), dtype=torch.uint8, device=dev)
+            rows = [2 * i + 1 for i in range(len(w.sessions))]
+
+            def run():
+                for l in range(case.L):
+                    nexus.suffix_attention(case.cache, case.d_pt, case.n_rows, case.max_pages,
+                                           case.kv, ql, q[l:l + 1], o[l:l + 1], lse[l:l + 1], HQ,
+                                           l, l + 1, rows=rows, split_kv=0, workspace=ws,
+                                           workspace_bytes=wsb, stream=stream)
+            ms = _time_back_to_back(run, stream, warmup, reps)
+            tf = case.flops(pct) / (ms * 1e-3) / 1e12
+            sufs.append({"pct": pct, "q_len": ql if len(ql) <= 2 else {"sum": n_tok},
+                         "splits": splits, "ms": ms, "ms_per_layer": ms / case.L,
+                         "tflops": tf, "frac": tf / peak_tc, "bound": "tensor",
+                         "peak": peak_tc, "peak_kind": f"bf16 burst (timed alone), {peak_kind}"})
+            del q, o, lse, ws
+        line["suffix_attention"] = sufs
+        st = nexus.device_status(stream)
+        if st != nexus.OK:
+            raise RuntimeError(f"device status after config {name}: {nexus.status_string(st)}")
+        if with_oracle:
+            T = max(case.kv)
+            R = max(max(v) for v in case.q_len.values())
+            tf, g, desc = _oracle_config_sample(T, R)
+            line["cpu_baseline"] = {"value": tf, "unit": "TFLOP/s", "cores": cpu_cores(),
+                                    "kind": "oracle", "sample": desc, "splice_gbs": g}
+        out[name] = line
+        del case
+        torch.cuda.empty_cache()
     return out
 
 
