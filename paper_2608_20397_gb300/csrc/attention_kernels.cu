@@ -86,9 +86,16 @@ struct Work {
   int seq, kv, layer_rel, split;
   int tok0[2], ntok[2], pos0[2];
   bool has_b;
+  bool skip;            // a split index past this pair's split count: no work, no writes
   int kt_begin, n_tiles;
 };
 
+// kKinds: pairs holding two query tiles and pairs holding one take their own
+// split counts (splits_pair / splits_single, a split-KV plan); otherwise every
+// pair takes `splits`. Kept apart at compile time: selecting the count per
+// pair raised the register count of the whole kernel (166 -> 168) and slowed
+// the re-prefill's loops by ~1.5 %.
+template <bool kKinds>
 __device__ __forceinline__ Work decode_work(const AttnLaunch& p) {
   Work w;
   const int rev = p.total_tiles - 1 - (int)blockIdx.x;   // deepest query tiles first
@@ -113,10 +120,33 @@ __device__ __forceinline__ Work decode_work(const AttnLaunch& p) {
   const int last = w.has_b ? 1 : 0;
   const int pos_last = w.pos0[last] + w.ntok[last] - 1;
   const int kt_total = pos_last / BN + 1;
-  const int per = (kt_total + p.splits - 1) / p.splits;
-  w.kt_begin = w.split * per;
-  w.n_tiles = max(0, min(kt_total, w.kt_begin + per) - w.kt_begin);
+  // The pair's key tiles spread evenly over its split count (split <= 32 and
+  // kt_total <= 2^24 keep the products below 2^30).
+  if constexpr (kKinds) {
+    const int s_this = w.has_b ? p.splits_pair : p.splits_single;
+    w.skip = w.split >= s_this;
+    w.kt_begin = w.split * kt_total / s_this;
+    w.n_tiles = w.skip ? 0 : (w.split + 1) * kt_total / s_this - w.kt_begin;
+  } else {
+    w.skip = false;
+    w.kt_begin = w.split * kt_total / p.splits;
+    w.n_tiles = (w.split + 1) * kt_total / p.splits - w.kt_begin;
+  }
   return w;
+}
+
+// Split count of the pair that owns packed token `tok` (the merge needs it per row).
+__device__ __forceinline__ int splits_of_token(const AttnLaunch& p, int tok) {
+  if (p.splits_pair == p.splits_single) return p.splits_pair;
+  int lo = 0, hi = p.n_seqs - 1;   // last sequence starting at or before tok
+  while (lo < hi) {
+    const int mid = (lo + hi + 1) >> 1;
+    if (p.seq[mid].q_off <= tok) lo = mid; else hi = mid - 1;
+  }
+  const AttnSeq& s = p.seq[lo];
+  const int pair = (tok - s.q_off) / p.tile_tokens / 2;
+  const int q_tiles = (s.q_len + p.tile_tokens - 1) / p.tile_tokens;
+  return 2 * pair + 1 < q_tiles ? p.splits_pair : p.splits_single;
 }
 
 // Zeroes V rows of keys [r0, 128) of one stage, so cache slots past kv_len
@@ -268,7 +298,7 @@ __device__ __forceinline__ void issue_pv_rem(uint32_t t_o, uint32_t t_s, uint64_
 // pairs holding rows that see fewer than 128 keys (see short_rows below); the
 // host gives all other pairs to the kShort = false kernel, which carries none of
 // that code (its presence alone slowed the loops of every step by 1-2 %).
-template <bool kSoftcap, bool kShort>
+template <bool kSoftcap, bool kShort, bool kKinds>
 __global__ void __launch_bounds__(kThreads, 1)
 attention_kernel(const __grid_constant__ AttnLaunch p, const __grid_constant__ AttnMaps maps) {
   extern __shared__ uint8_t smem_raw[];
@@ -283,7 +313,8 @@ attention_kernel(const __grid_constant__ AttnLaunch p, const __grid_constant__ A
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
-  const Work w = decode_work(p);
+  const Work w = decode_work<kKinds>(p);
+  if (w.skip) return;   // before any barrier, TMEM or global memory use
   const AttnSeq sq = p.seq[w.seq];
   const int G = p.group;
   const int layer = p.layer_begin + w.layer_rel;
@@ -336,6 +367,12 @@ attention_kernel(const __grid_constant__ AttnLaunch p, const __grid_constant__ A
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
   const bool vt = p.v_transposed != 0;
+  // Launched with programmatic stream serialization: the setup above (shared
+  // memory, barriers, TMEM) overlaps the previous kernel's tail; nothing in
+  // global memory is touched before that kernel has completed (the partials a
+  // previous merge still reads, the Q / K / V it wrote).
+  griddep_wait();
+  griddep_launch_dependents();
 
   if (warp == kProducerWarp) {
     // ------------------------------------------------------ TMA producer
@@ -745,15 +782,26 @@ attention_kernel(const __grid_constant__ AttnLaunch p, const __grid_constant__ A
 
 // Merge of split-KV partials: one warp per (layer, token, head) row. Lane s
 // holds split s's LSE; the max and the weight sum are warp-shuffle
-// reductions, then every lane accumulates its four columns over the splits,
-// eight splits' loads in flight at a time (they are independent; a loop of one
-// load at a time waited out an L2 round trip per split).
+// reductions, then every lane accumulates its four columns over the splits.
+// Every split writes every row it owns (zeros and an LSE of -inf where it saw
+// no key), so the first 16 splits' partial rows are loaded together with the
+// LSE, before the weights are known: one memory round trip for up to 16 splits.
 __global__ void __launch_bounds__(128) combine_kernel(const __grid_constant__ AttnLaunch p) {
+  griddep_wait();   // the attention grid's partials are complete and visible
+  griddep_launch_dependents();
   const int64_t rows = (int64_t)p.n_layers_call * p.n_tok * p.n_q_heads;
   const int64_t row = (int64_t)blockIdx.x * 4 + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
   if (row >= rows) return;
-  const float l_s = lane < p.splits ? p.part_lse[(int64_t)lane * rows + row] : -INFINITY;
+  const int splits = splits_of_token(p, static_cast<int>((row / p.n_q_heads) % p.n_tok));
+  constexpr int kBatch = 16;
+  float4 v[kBatch];
+  const float l_s = lane < splits ? __ldcg(p.part_lse + (int64_t)lane * rows + row) : -INFINITY;
+#pragma unroll
+  for (int k = 0; k < kBatch; ++k)
+    v[k] = k < splits
+               ? __ldcg(reinterpret_cast<const float4*>(p.part_o + ((int64_t)k * rows + row) * D) + lane)
+               : make_float4(0.f, 0.f, 0.f, 0.f);
   float mx = l_s;
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
@@ -762,21 +810,19 @@ __global__ void __launch_bounds__(128) combine_kernel(const __grid_constant__ At
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) wsum += __shfl_xor_sync(0xffffffffu, wsum, o);
   float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-  for (int s0 = 0; s0 < p.splits; s0 += 8) {
-    float4 v[8];
-    float ws[8];
+  for (int s0 = 0; s0 < splits; s0 += kBatch) {
+    if (s0 > 0) {
 #pragma unroll
-    for (int k = 0; k < 8; ++k) {
-      const int s = s0 + k;
-      ws[k] = __shfl_sync(0xffffffffu, w, s & 31);
-      v[k] = (s < p.splits && ws[k] != 0.f)
-                 ? __ldcg(reinterpret_cast<const float4*>(p.part_o + ((int64_t)s * rows + row) * D) + lane)
-                 : make_float4(0.f, 0.f, 0.f, 0.f);
+      for (int k = 0; k < kBatch; ++k)
+        v[k] = s0 + k < splits
+                   ? __ldcg(reinterpret_cast<const float4*>(p.part_o + ((int64_t)(s0 + k) * rows + row) * D) + lane)
+                   : make_float4(0.f, 0.f, 0.f, 0.f);
     }
 #pragma unroll
-    for (int k = 0; k < 8; ++k) {
-      if (s0 + k < p.splits && ws[k] != 0.f) {
-        acc.x += ws[k] * v[k].x; acc.y += ws[k] * v[k].y; acc.z += ws[k] * v[k].z; acc.w += ws[k] * v[k].w;
+    for (int k = 0; k < kBatch; ++k) {
+      const float ws = __shfl_sync(0xffffffffu, w, (s0 + k) & 31);
+      if (s0 + k < splits && ws != 0.f) {
+        acc.x += ws * v[k].x; acc.y += ws * v[k].y; acc.z += ws * v[k].z; acc.w += ws * v[k].w;
       }
     }
   }
@@ -808,23 +854,49 @@ cudaError_t launch_wait_selftest(uint64_t budget_ns, cudaStream_t stream) {
 cudaError_t launch_attention(const AttnLaunch& p, const AttnMaps& maps, cudaStream_t stream) {
   if (p.total_tiles <= 0 || p.n_layers_call <= 0) return cudaSuccess;
   static_assert(kSmemBytes <= 227 * 1024, "shared memory budget");
-  auto kernel = p.softcap_out > 0.f
-                    ? (p.short_rows ? attention_kernel<true, true> : attention_kernel<true, false>)
-                    : (p.short_rows ? attention_kernel<false, true> : attention_kernel<false, false>);
+  const bool kinds = p.splits_pair != p.splits_single;
+  void (*kernel)(const AttnLaunch, const AttnMaps);
+  if (p.softcap_out > 0.f)
+    kernel = p.short_rows ? (kinds ? attention_kernel<true, true, true> : attention_kernel<true, true, false>)
+                          : (kinds ? attention_kernel<true, false, true> : attention_kernel<true, false, false>);
+  else
+    kernel = p.short_rows ? (kinds ? attention_kernel<false, true, true> : attention_kernel<false, true, false>)
+                          : (kinds ? attention_kernel<false, false, true> : attention_kernel<false, false, false>);
   cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        (int)kSmemBytes);
   if (e != cudaSuccess) return e;
   const dim3 grid((unsigned)p.total_tiles, (unsigned)p.n_kv_heads,
                   (unsigned)(p.n_layers_call * p.splits));
-  kernel<<<grid, kThreads, kSmemBytes, stream>>>(p, maps);
-  return cudaGetLastError();
+  // Programmatic stream serialization: the CTAs may start (and set up) while
+  // the previous kernel of the stream finishes; they wait for it before any
+  // global memory access.
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = kSmemBytes;
+  cfg.stream = stream;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, p, maps);
 }
 
 cudaError_t launch_attn_combine(const AttnLaunch& p, cudaStream_t stream) {
   const int64_t rows = (int64_t)p.n_layers_call * p.n_tok * p.n_q_heads;
   if (rows <= 0) return cudaSuccess;
-  combine_kernel<<<(unsigned)((rows + 3) / 4), 128, 0, stream>>>(p);
-  return cudaGetLastError();
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)((rows + 3) / 4));
+  cfg.blockDim = dim3(128);
+  cfg.dynamicSmemBytes = 0;
+  cfg.stream = stream;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, combine_kernel, p);
 }
 
 cudaError_t attention_take_timeout(unsigned int* flag, cudaStream_t stream) {

@@ -109,6 +109,10 @@ struct AttnLaunch {
   AttnSeq seq[kMaxSeqs];
   int32_t pair0[kMaxSeqs];  // first tile pair of each sequence in this launch
   int32_t short_rows;       // this launch's tile pairs hold rows that see fewer than 128 keys
+  // Key splits of a pair holding two query tiles / one query tile (both at
+  // most `splits`, which sizes the grid and the partials).
+  int32_t splits_pair;
+  int32_t splits_single;
 };
 
 struct AttnMaps {

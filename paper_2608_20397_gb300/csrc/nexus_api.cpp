@@ -289,7 +289,9 @@ int slb_grid(int32_t n_tools, int32_t n_queries, int32_t* per_out) {
 struct AttnPlan {
   int32_t total_tiles = 0;
   int32_t n_tok = 0;
-  int32_t splits = 1;
+  int32_t splits = 1;          // grid and partials: the larger of the two below
+  int32_t splits_pair = 1;     // key splits of a pair holding two query tiles
+  int32_t splits_single = 1;   // ... holding one query tile
   int32_t kt_max = 0;
 };
 
@@ -304,6 +306,8 @@ nexus_status plan_attention(int32_t n_seqs, const int32_t* kv_len, const int32_t
   AttnPlan pl;
   int64_t tok = 0, tiles = 0;
   double key_tiles = 0.0;   // key tiles over all CTAs of one KV head (no split)
+  int64_t n_pair = 0, n_single = 0;   // pairs holding two / one query tile
+  int32_t kt_pair = 0, kt_single = 0; // their largest key-tile counts
   for (int32_t s = 0; s < n_seqs; ++s) {
     if (q_len[s] < 0 || kv_len[s] < q_len[s]) return NEXUS_EINVAL;
     tok += q_len[s];
@@ -313,7 +317,10 @@ nexus_status plan_attention(int32_t n_seqs, const int32_t* kv_len, const int32_t
     if (q_len[s] > 0) pl.kt_max = std::max(pl.kt_max, (kv_len[s] + 127) / 128);
     for (int32_t k = 0; k < pairs; ++k) {
       const int64_t last_tok = std::min<int64_t>(q_len[s], (2 * k + 2) * int64_t{tile_tokens}) - 1;
-      key_tiles += static_cast<double>((kv_len[s] - q_len[s] + last_tok) / 128 + 1);
+      const int32_t kt = static_cast<int32_t>((kv_len[s] - q_len[s] + last_tok) / 128 + 1);
+      key_tiles += static_cast<double>(kt);
+      if (2 * k + 1 < q_tiles) { ++n_pair; kt_pair = std::max(kt_pair, kt); }
+      else { ++n_single; kt_single = std::max(kt_single, kt); }
     }
   }
   if (tok > 0x7FFFFFFF || tiles > 0x7FFFFFFF) return NEXUS_ERANGE;
@@ -350,9 +357,36 @@ nexus_status plan_attention(int32_t n_seqs, const int32_t* kv_len, const int32_t
       }
       if (best_cost > 0.9 * c1) best = 1;
     }
-    pl.splits = best;
+    pl.splits = pl.splits_pair = pl.splits_single = best;
+    // Split, all CTAs in one wave, pairs of both kinds present: a pair holding
+    // one query tile runs a key-tile step in ~0.87 of a two-tile pair's time and
+    // ends ~3 steps sooner (one tile to write back), so it takes fewer splits
+    // over longer key ranges and the two kinds end together. Measured on the c5
+    // suffix (9 splits each): two-tile pairs end at ~63 us, one-tile pairs at ~52.
+    const int64_t units = static_cast<int64_t>(n_kv_heads) * std::max(1, n_layers_call);
+    if (best > 1 && n_pair > 0 && n_single > 0 && ctas * best <= sms) {
+      constexpr double kSingleStep = 0.87, kPairFixed = 6.1, kSingleFixed = 3.2;
+      auto span = [&](int sp, int ss) {
+        const double tp = std::ceil(static_cast<double>(kt_pair) / sp) + kPairFixed;
+        const double ts = kSingleStep * std::ceil(static_cast<double>(kt_single) / ss) + kSingleFixed;
+        const int sm = std::max(sp, ss);
+        return std::max(tp, ts) + (3.0 + sm * rows * (kHeadDim * 4 + 4) / kMergeBytesPerUs) / kStepUs;
+      };
+      double best_span = span(best, best);
+      for (int sp = 1; sp <= std::min<int>(kMaxSplits, kt_pair); ++sp)
+        for (int ss = 1; ss <= std::min<int>(kMaxSplits, kt_single); ++ss) {
+          if (units * (n_pair * sp + n_single * ss) > sms) continue;
+          const double c = span(sp, ss);
+          if (c < best_span - 1e-9) {
+            best_span = c;
+            pl.splits_pair = sp;
+            pl.splits_single = ss;
+          }
+        }
+      pl.splits = std::max(pl.splits_pair, pl.splits_single);
+    }
   } else {
-    pl.splits = std::min(split_kv, kMaxSplits);
+    pl.splits = pl.splits_pair = pl.splits_single = std::min(split_kv, kMaxSplits);
   }
   *out = pl;
   return NEXUS_OK;
@@ -408,6 +442,8 @@ nexus_status attention_impl(const nexus_kv_cache* c, const int32_t* d_pt, int32_
   p->n_layers_call = le - lb;
   p->n_seqs = n_seqs;
   p->splits = pl.splits;
+  p->splits_pair = pl.splits_pair;
+  p->splits_single = pl.splits_single;
   p->v_transposed = c->v_transposed;
   p->total_tiles = pl.total_tiles;
   p->scale_log2 = static_cast<float>(1.4426950408889634 / std::sqrt(static_cast<double>(kHeadDim)));

@@ -66,6 +66,21 @@ __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, uint64_
   }
 }
 
+// ------------------------------------------- programmatic dependent launch
+// Waits until every grid this one depends on (the previous kernel of the
+// stream) has completed and its memory is visible; a no-op for a kernel
+// launched without programmatic stream serialization. Every global memory
+// access of a kernel launched with it must come after this wait.
+__device__ __forceinline__ void griddep_wait() {
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+}
+// Lets the next kernel of the stream (if launched with programmatic stream
+// serialization) start its CTAs once every CTA of this grid has issued this or
+// exited; the next kernel's own griddep_wait still waits for this grid's end.
+__device__ __forceinline__ void griddep_launch_dependents() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
 // ------------------------------------------------------------------- TMA
 __device__ __forceinline__ void prefetch_tmap(const CUtensorMap* m) {
   asm volatile("prefetch.tensormap [%0];" ::"l"(m) : "memory");
