@@ -140,7 +140,7 @@ class C5:
     """Device-resident c5 workload and the library calls of one step (also used
     with the c3 workload, whose cache keeps V token-innermost, for captures)."""
 
-    def __init__(self, dev, n_layers=48, name="c5"):
+    def __init__(self, dev, n_layers=48, name="c5", prefill=True):
         import torch
 
         from paper_2608_20397_gb300 import nexus
@@ -186,9 +186,11 @@ class C5:
         h_pt[1] = new_pt
         self.h_pt = h_pt
         self.d_pt = torch.as_tensor(h_pt, device=dev)
-        self.q_pre = randn_bf16((L, self.n_past, HQ, D), 800, dev)
-        self.o_pre = torch.empty_like(self.q_pre)
-        self.lse_pre = torch.empty((L, self.n_past, HQ), dtype=torch.float32, device=dev)
+        # the re-prefill's Q and O (16 GB each at 48 layers): only where they are used
+        self.q_pre = randn_bf16((L, self.n_past, HQ, D), 800, dev) if prefill else None
+        self.o_pre = torch.empty_like(self.q_pre) if prefill else None
+        self.lse_pre = (torch.empty((L, self.n_past, HQ), dtype=torch.float32, device=dev)
+                        if prefill else None)
         self.q_suf = randn_bf16((L, self.R_split, HQ, D), 900, dev)
         self.o_suf = torch.empty_like(self.q_suf)
         self.lse_suf = torch.empty((L, self.R_split, HQ), dtype=torch.float32, device=dev)
@@ -199,7 +201,9 @@ class C5:
         self.splice_bytes = 8192.0 * self.splice_rows * L
         self.flops_pre = attn_flops(self.n_past, self.n_past, L)
         self.flops_suf = attn_flops(self.T, self.R_split, L)
-        self.launches_per_step = 1 + L + L * (2 if self.splits > 1 else 1)
+        # per layer: the re-prefill's plain grid plus the grid of its first tile
+        # pairs (rows that see fewer than 128 keys); the suffix plus its merge
+        self.launches_per_step = 1 + 2 * L + L * (2 if self.splits > 1 else 1)
 
     # library calls of one step; optional events bracket the splice and the re-prefill
     def step(self, stream, ev=None, q_pre=None, o_pre=None):
@@ -343,7 +347,8 @@ def main():
     nexus.lib()
     if args.profile is None and args.workload != "c5":
         raise SystemExit("the timed step is the c5 workload; --workload only applies to --profile")
-    wl = C5(dev, args.layers, args.workload)
+    wl = C5(dev, args.layers, args.workload,
+            prefill=args.profile in (None, "reprefill", "reprefill-softcap"))
     stream = torch.cuda.current_stream()
     peaks, peak_kind = measured_peaks()
 
