@@ -151,6 +151,7 @@ struct QkvLaunch {
   int32_t total_tiles;      // m_tiles * n_tiles
   int32_t n_seqs;
   int32_t short_tiles;      // n_tok <= 64: one-head tiles, 64 token rows per stage
+  int32_t pair_split;       // short tiles: two CTAs (a cluster) per tile split the hidden dim
   float inv_freq_hi[kHeadDim / 2];   // theta_i / pi = hi + lo
   float inv_freq_lo[kHeadDim / 2];
   AttnSeq seq[kMaxSeqs];

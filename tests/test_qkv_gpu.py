@@ -259,6 +259,28 @@ def test_qkv_short_suffix_ragged_sequences(dev):
     c.check_untouched()
 
 
+@pytest.mark.parametrize("hidden,gptj", [(256, True), (448, False), (HIDDEN, True)])
+def test_qkv_short_pair_split_hidden(dev, hidden, gptj):
+    # Up to 64 tokens each head's tile is shared by a pair of CTAs that split the
+    # hidden dimension and add their partial sums over distributed shared memory:
+    # the smallest split (two stages, the second partly past the hidden size), an
+    # odd stage count, and the bench's width with GPT-J pairs; varlen with a
+    # one-token sequence; two runs bit-identical.
+    c = QkvCase(dev, [700, 9000, 33], [1, 40, 23], hidden, gptj=gptj, seed=34 + hidden)
+    c.run()
+    torch.cuda.synchronize()
+    c.check(what=f"pair split hidden {hidden} gptj={gptj}")
+    c.check_untouched()
+    q1 = c.q.clone()
+    k1, v1 = c.kp.clone(), c.vp.clone()
+    c.run()
+    torch.cuda.synchronize()
+    assert torch.equal(q1.view(torch.int16), c.q.view(torch.int16))
+    assert torch.equal(k1.view(torch.int16), c.kp.view(torch.int16))
+    assert torch.equal(v1.view(torch.int16), c.vp.view(torch.int16))
+    assert nexus.device_status() == nexus.OK
+
+
 def test_qkv_65_tokens_take_long_tiles(dev):
     c = QkvCase(dev, [300], [65], 512, seed=33)
     c.run()
