@@ -590,9 +590,9 @@ attention_kernel(const __grid_constant__ AttnLaunch p, const __grid_constant__ A
           const float2 zb = ffma2(b, half, half);
           const float2 zp = fmul2(za, zb);
           const float r = rcp_approx(zp.x * zp.y);
-          const float2 rp = make_float2(r * zp.y, r * zp.x);
-          const float2 ta = fadd2(fmul2(rp, zb), mone);
-          const float2 tb = fadd2(fmul2(rp, za), mone);
+          const float2 rp = fmul2(make_float2(r, r), make_float2(zp.y, zp.x));
+          const float2 ta = ffma2(rp, zb, mone);
+          const float2 tb = ffma2(rp, za, mone);
           s[c] = ta.x;
           s[c + 1] = ta.y;
           s[c + 2] = tb.x;
