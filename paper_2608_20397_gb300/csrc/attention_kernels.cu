@@ -96,7 +96,56 @@ struct Work {
 // pair raised the register count of the whole kernel (166 -> 168) and slowed
 // the re-prefill's loops by ~1.5 %.
 template <bool kKinds>
-__device__ __forceinline__ Work decode_work(const AttnLaunch& p) {
+__device__ __forceinline__ Work decode_work(const AttnLaunch& p);
+
+// Split plans with per-kind counts: x enumerates exactly the (pair, split)
+// CTAs of every sequence, deepest first, so no CTA is launched past its
+// pair's split count.
+template <>
+__device__ __forceinline__ Work decode_work<true>(const AttnLaunch& p) {
+  Work w;
+  const int rev = p.cta_prefix[p.n_seqs] - 1 - (int)blockIdx.x;
+  int lo = 0, hi = p.n_seqs - 1;
+  while (lo < hi) {
+    const int mid = (lo + hi + 1) >> 1;
+    if (p.cta_prefix[mid] <= rev) lo = mid; else hi = mid - 1;
+  }
+  w.seq = lo;
+  const AttnSeq& s = p.seq[lo];
+  const int q_tiles = (s.q_len + p.tile_tokens - 1) / p.tile_tokens;
+  const int local = rev - p.cta_prefix[lo];
+  const int full = q_tiles / 2;
+  int pair;
+  if (local < full * p.splits_pair) {
+    pair = local / p.splits_pair;
+    w.split = local % p.splits_pair;
+  } else {
+    pair = full;
+    w.split = local - full * p.splits_pair;
+  }
+  w.kv = blockIdx.y;
+  w.layer_rel = blockIdx.z;
+  w.has_b = 2 * pair + 1 < q_tiles;
+  for (int x = 0; x < 2; ++x) {
+    w.tok0[x] = (2 * pair + x) * p.tile_tokens;
+    w.ntok[x] = max(0, min(p.tile_tokens, s.q_len - w.tok0[x]));
+    w.pos0[x] = s.kv_len - s.q_len + w.tok0[x];
+  }
+  const int last = w.has_b ? 1 : 0;
+  const int pos_last = w.pos0[last] + w.ntok[last] - 1;
+  const int kt_total = pos_last / BN + 1;
+  // key tiles spread evenly over the pair's own split count (split <= 32 and
+  // kt_total <= 2^24 keep the products below 2^30)
+  const int s_this = w.has_b ? p.splits_pair : p.splits_single;
+  w.skip = false;
+  w.kt_begin = w.split * kt_total / s_this;
+  w.n_tiles = (w.split + 1) * kt_total / s_this - w.kt_begin;
+  return w;
+}
+
+template <>
+__device__ __forceinline__ Work decode_work<false>(const AttnLaunch& p) {
+  constexpr bool kKinds = false;
   Work w;
   const int rev = p.total_tiles - 1 - (int)blockIdx.x;   // deepest query tiles first
   int lo = 0, hi = p.n_seqs - 1;
@@ -854,7 +903,7 @@ cudaError_t launch_wait_selftest(uint64_t budget_ns, cudaStream_t stream) {
 cudaError_t launch_attention(const AttnLaunch& p, const AttnMaps& maps, cudaStream_t stream) {
   if (p.total_tiles <= 0 || p.n_layers_call <= 0) return cudaSuccess;
   static_assert(kSmemBytes <= 227 * 1024, "shared memory budget");
-  const bool kinds = p.splits_pair != p.splits_single;
+  const bool kinds = p.splits_pair != p.splits_single && p.cta_prefix[p.n_seqs] > 0;
   void (*kernel)(const AttnLaunch, const AttnMaps);
   if (p.softcap_out > 0.f)
     kernel = p.short_rows ? (kinds ? attention_kernel<true, true, true> : attention_kernel<true, true, false>)
@@ -865,8 +914,10 @@ cudaError_t launch_attention(const AttnLaunch& p, const AttnMaps& maps, cudaStre
   cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        (int)kSmemBytes);
   if (e != cudaSuccess) return e;
-  const dim3 grid((unsigned)p.total_tiles, (unsigned)p.n_kv_heads,
-                  (unsigned)(p.n_layers_call * p.splits));
+  const dim3 grid = kinds ? dim3((unsigned)p.cta_prefix[p.n_seqs], (unsigned)p.n_kv_heads,
+                                 (unsigned)p.n_layers_call)
+                         : dim3((unsigned)p.total_tiles, (unsigned)p.n_kv_heads,
+                                (unsigned)(p.n_layers_call * p.splits));
   // Programmatic stream serialization: the CTAs may start (and set up) while
   // the previous kernel of the stream finishes; they wait for it before any
   // global memory access.

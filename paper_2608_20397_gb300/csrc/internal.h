@@ -113,6 +113,10 @@ struct AttnLaunch {
   // most `splits`, which sizes the grid and the partials).
   int32_t splits_pair;
   int32_t splits_single;
+  // Split plans with per-kind counts: the grid's x runs over exactly the
+  // (tile pair, split) CTAs of every sequence; cta_prefix[s] is the first of
+  // sequence s (kinds launches only).
+  int32_t cta_prefix[kMaxSeqs + 1];
 };
 
 struct AttnMaps {

@@ -364,7 +364,10 @@ nexus_status plan_attention(int32_t n_seqs, const int32_t* kv_len, const int32_t
     // over longer key ranges and the two kinds end together. Measured on the c5
     // suffix (9 splits each): two-tile pairs end at ~63 us, one-tile pairs at ~52.
     const int64_t units = static_cast<int64_t>(n_kv_heads) * std::max(1, n_layers_call);
-    if (best > 1 && n_pair > 0 && n_single > 0 && ctas * best <= sms) {
+    bool short_rows = false;   // tile pairs whose rows see fewer than 128 keys: uniform splits
+    for (int32_t s = 0; s < n_seqs; ++s)
+      short_rows = short_rows || (q_len[s] > 0 && kv_len[s] - q_len[s] < 127);
+    if (best > 1 && n_pair > 0 && n_single > 0 && ctas * best <= sms && !short_rows) {
       constexpr double kSingleStep = 0.87, kPairFixed = 6.1, kSingleFixed = 3.2;
       auto span = [&](int sp, int ss) {
         const double tp = std::ceil(static_cast<double>(kt_pair) / sp) + kPairFixed;
@@ -497,6 +500,17 @@ nexus_status attention_impl(const nexus_kv_cache* c, const int32_t* d_pt, int32_
   }
   p->tile_prefix[n_seqs] = tiles;
   p->total_tiles = tiles;
+  if (pl.splits_pair != pl.splits_single) {
+    // per-kind split counts (the planner gives them only without short rows):
+    // the grid enumerates each pair's own (pair, split) CTAs
+    int32_t ctas = 0;
+    for (int32_t s = 0; s < n_seqs; ++s) {
+      p->cta_prefix[s] = ctas;
+      const int32_t q_tiles = (q_len[s] + tt - 1) / tt;
+      ctas += (q_tiles / 2) * pl.splits_pair + (q_tiles % 2) * pl.splits_single;
+    }
+    p->cta_prefix[n_seqs] = ctas;
+  }
 
   AttnMaps maps;
   const uint64_t tok_stride = static_cast<uint64_t>(n_q_heads) * kHeadDim * 2;
