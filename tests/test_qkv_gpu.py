@@ -287,3 +287,61 @@ def test_qkv_65_tokens_take_long_tiles(dev):
     torch.cuda.synchronize()
     c.check(what="65 tokens")
     c.check_untouched()
+
+
+def test_recompute_then_attention_back_to_back(dev):
+    """The re-decode of a layer as a model runs it: fresh Q/K/V, then the suffix
+    attention reading them, then the next recompute overwriting them, all on one
+    stream with no synchronisation. The launches overlap their setup with the
+    previous kernel (programmatic dependent launch) and must still read only
+    completed inputs and not overwrite inputs still being read: the attention
+    output equals the one of the same calls synchronised after each step, bit for
+    bit, and the oracle's on the recomputed Q, K and V."""
+    kv, ql = [3000], [64]
+    c = QkvCase(dev, kv, ql, HIDDEN, seed=61, n_layers=2, layer=1)
+    x1, x2 = c.x.clone(), randn_bf16(c.x.shape, 62, dev)
+    need, _ = nexus.attention_workspace_size(kv, ql, 40, 8, 1, 0)
+    ws = torch.empty(max(16, need), dtype=torch.uint8, device=dev)
+
+    def attend(o, lse, stream=None):
+        nexus.suffix_attention(c.cache, c.d_pt, 1, c.max_pages, kv, ql, c.q[None], o, lse, 40,
+                               c.layer, c.layer + 1, split_kv=0, workspace=ws,
+                               workspace_bytes=need, stream=stream)
+
+    k0, v0 = c.kp.clone(), c.vp.clone()
+    # synchronised after every step
+    c.x = x1
+    c.run()
+    torch.cuda.synchronize()
+    q1, kp1, vp1 = c.q.clone(), c.kp.clone(), c.vp.clone()
+    o_ref = torch.empty((1, 64, 40, 128), dtype=torch.bfloat16, device=dev)
+    l_ref = torch.empty((1, 64, 40), dtype=torch.float32, device=dev)
+    attend(o_ref, l_ref)
+    torch.cuda.synchronize()
+    # back to back on one stream
+    c.kp.copy_(k0)
+    c.vp.copy_(v0)
+    s = torch.cuda.Stream()
+    o = torch.full_like(o_ref, float("nan"))
+    l = torch.full_like(l_ref, float("nan"))
+    torch.cuda.synchronize()
+    with torch.cuda.stream(s):   # three library launches back to back, nothing between
+        c.x = x1
+        c.run(stream=s)
+        attend(o, l, stream=s)
+        c.x = x2
+        c.run(stream=s)
+    s.synchronize()
+    assert nexus.device_status() == nexus.OK
+    assert torch.equal(o.view(torch.int16), o_ref.view(torch.int16))
+    assert torch.equal(l, l_ref)
+    # and the oracle on the recomputed rows (sampled)
+    rows = np.array([0, 1, 31, 62, 63])
+    pos = np.arange(kv[0] - ql[0], kv[0])
+    pg = torch.as_tensor(c.h_pt[0][np.arange(kv[0]) // 16], device=dev).long()
+    sl = torch.arange(kv[0], device=dev) % 16
+    k_all = kp1[c.layer][pg, :, sl, :]
+    v_all = vp1[c.layer][pg, :, sl, :]
+    want, want_l = oracle.attention(f64(q1[rows]), f64(k_all), f64(v_all), pos[rows], 5)
+    from gpu_cases import assert_attn_close
+    assert_attn_close(f64(o[0, rows]), want, f64(l[0, rows]), want_l, "recompute then attention")
