@@ -4,7 +4,7 @@
 // into the token's slot of the paged cache (either V layout, Sec. V-B).
 //
 // Persistent CTAs, one per SM, walk output tiles of 128 tokens x 256 features
-// (two heads) in bands of group_m token tiles, the token tile fastest inside a
+// (two heads) in bands of group_m (24) token tiles, the token tile fastest inside a
 // band: the tiles in flight at any time share a few weight tiles and the
 // band's token rows, which stay in L2, so DRAM sees each weight tile once per
 // band rather than once per wave. Up to 64 tokens (a short re-decoded suffix)
