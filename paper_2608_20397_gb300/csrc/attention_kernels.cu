@@ -784,6 +784,53 @@ attention_kernel(const __grid_constant__ AttnLaunch p, const __grid_constant__ A
     const int head = w.kv * G + (r % G);
     const int64_t row = ((int64_t)w.layer_rel * p.n_tok + tok) * p.n_q_heads + head;
     const int64_t rows_per_split = (int64_t)p.n_layers_call * p.n_tok * p.n_q_heads;
+    if constexpr (kKinds) {
+      // Split plans: the float32 partial rows go through shared memory so that
+      // each is written as one coalesced 512-byte store; a thread storing its
+      // own row scattered every warp store over 32 rows (half sectors), and a
+      // two-tile CTA spent ~6 us on it. Each warp stages its own 32 rows (16 KB,
+      // 16-byte chunks XOR-swizzled by the row): tile A in the K ring (free once
+      // its last P V product completed: every S product precedes it), tile B in
+      // the V ring (free once its own last P V completed).
+      if (x < n_q) {
+        const int lw = r & 31;
+        const uint32_t stage = sbase + (x == 0 ? OFF_K : OFF_V) + (warp & 3) * 16384;
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          uint32_t v[32];
+          if (have_o) {
+            tmem_ld32(t_o + q * 32, v);
+            tmem_ld_wait();
+          }
+#pragma unroll
+          for (int c = 0; c < 8; ++c) {
+            const int chunk = q * 8 + c;
+            const float4 f = have_o ? make_float4(__uint_as_float(v[4 * c]) * inv_l,
+                                                  __uint_as_float(v[4 * c + 1]) * inv_l,
+                                                  __uint_as_float(v[4 * c + 2]) * inv_l,
+                                                  __uint_as_float(v[4 * c + 3]) * inv_l)
+                                    : make_float4(0.f, 0.f, 0.f, 0.f);
+            st_shared_v4(stage + lw * 512 + ((chunk ^ lw) & 31) * 16, __float_as_uint(f.x),
+                         __float_as_uint(f.y), __float_as_uint(f.z), __float_as_uint(f.w));
+          }
+        }
+        __syncwarp();
+        // row i of the warp: lane i's row index and validity, broadcast
+        float* const base = p.part_o + (int64_t)w.split * rows_per_split * D + lane * 4;
+        const unsigned valid_mask = __ballot_sync(0xffffffffu, row_valid);
+        const uint32_t row_lo = static_cast<uint32_t>(row), row_hi = static_cast<uint32_t>(row >> 32);
+#pragma unroll 4
+        for (int i = 0; i < 32; ++i) {
+          const uint32_t lo = __shfl_sync(0xffffffffu, row_lo, i);
+          const uint32_t hi = __shfl_sync(0xffffffffu, row_hi, i);
+          if (!((valid_mask >> i) & 1u)) continue;   // the same for the whole warp
+          const int64_t row_i = static_cast<int64_t>((static_cast<uint64_t>(hi) << 32) | lo);
+          const float4 val = ld_shared_v4f(stage + i * 512 + ((lane ^ i) & 31) * 16);
+          __stcg(reinterpret_cast<float4*>(base + row_i * D), val);
+        }
+        if (row_valid) p.part_lse[(int64_t)w.split * rows_per_split + row] = lse;
+      }
+    } else {
 #pragma unroll
     for (int q = 0; q < 4; ++q) {
       uint32_t v[32];
@@ -820,6 +867,7 @@ attention_kernel(const __grid_constant__ AttnLaunch p, const __grid_constant__ A
       } else {
         p.part_lse[(int64_t)w.split * rows_per_split + row] = lse;
       }
+    }
     }
   }
 
@@ -903,7 +951,7 @@ cudaError_t launch_wait_selftest(uint64_t budget_ns, cudaStream_t stream) {
 cudaError_t launch_attention(const AttnLaunch& p, const AttnMaps& maps, cudaStream_t stream) {
   if (p.total_tiles <= 0 || p.n_layers_call <= 0) return cudaSuccess;
   static_assert(kSmemBytes <= 227 * 1024, "shared memory budget");
-  const bool kinds = p.splits_pair != p.splits_single && p.cta_prefix[p.n_seqs] > 0;
+  const bool kinds = p.splits > 1 && !p.short_rows && p.cta_prefix[p.n_seqs] > 0;
   void (*kernel)(const AttnLaunch, const AttnMaps);
   if (p.softcap_out > 0.f)
     kernel = p.short_rows ? (kinds ? attention_kernel<true, true, true> : attention_kernel<true, true, false>)

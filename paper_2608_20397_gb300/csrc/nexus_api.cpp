@@ -500,9 +500,9 @@ nexus_status attention_impl(const nexus_kv_cache* c, const int32_t* d_pt, int32_
   }
   p->tile_prefix[n_seqs] = tiles;
   p->total_tiles = tiles;
-  if (pl.splits_pair != pl.splits_single) {
-    // per-kind split counts (the planner gives them only without short rows):
-    // the grid enumerates each pair's own (pair, split) CTAs
+  if (pl.splits > 1 && n_short == 0) {
+    // split plans without short-row pairs (per-kind split counts occur only
+    // there): the grid enumerates each pair's own (pair, split) CTAs
     int32_t ctas = 0;
     for (int32_t s = 0; s < n_seqs; ++s) {
       p->cta_prefix[s] = ctas;
