@@ -140,6 +140,32 @@ def test_split_kv_uneven_pairs():
     _check(ks, vs, q, o, lse, kv, ql, 5, what="uneven pairs")
 
 
+# A tile pair holding one query tile, under a split plan, runs its key range in
+# both tile slots (even key tiles in slot A, odd in slot B) and merges the two
+# before writing its partial rows. Cases: the last CTA with key tiles 7 | 8,
+# where rows 1016..1023 see no key of tile 8 (slot B empty for them); three
+# tiles a CTA (the ragged tile in slot A); long ranges with a soft cap; a
+# sequence holding only a one-tile pair; transposed V.
+@pytest.mark.parametrize("kv,ql,split,vt,cap", [
+    (1030, 64, 5, False, None), (1030, 64, 4, True, None), (5000, 64, 3, False, 30.0),
+    (4100, 14, 2, True, None), (4100, 14, 7, False, 20.0), (2222, 110, 6, True, 50.0)])
+def test_split_kv_one_tile_pair_both_slots(kv, ql, split, vt, cap):
+    kv, ql = [kv], [ql]
+    cache, d_pt, mp, ks, vs, q = _direct_case(kv, ql, vt=vt, seed=kv[0] + split)
+    if cap is None:
+        o, lse = _run(cache, d_pt, mp, kv, ql, q, 40, 1, split_kv=split)
+    else:
+        o = torch.full_like(q, float("nan"))
+        lse = torch.full(q.shape[:3], float("nan"), dtype=torch.float32, device=DEV)
+        nbytes, _ = nexus.attention_workspace_size(kv, ql, 40, 8, 1, split)
+        ws = torch.empty(max(nbytes, 16), dtype=torch.uint8, device=DEV)
+        nexus.suffix_attention_softcap(cache, d_pt, 1, mp, kv, ql, q, o, lse, 40, 0, 1,
+                                       split_kv=split, workspace=ws, workspace_bytes=nbytes,
+                                       softcap=cap)
+        assert nexus.device_status() == nexus.OK
+    _check(ks, vs, q, o, lse, kv, ql, 5, what=f"one-tile pair split {split}", softcap=cap)
+
+
 def test_reprefill_equals_textbook_causal():
     T = 600
     cache, d_pt, mp, ks, vs, q = _direct_case([T], [T], seed=13)
