@@ -5,16 +5,18 @@
 // One CTA owns two 128-row query tiles (A and B) of one KV head. Rows are
 // (token, head in the GQA group) pairs, 128 / group tokens x group heads, so
 // every K/V tile brought into shared memory serves all query heads that read
-// it, twice. Per CTA (320 threads):
+// it, twice. Per CTA (352 threads):
 //
 //   warp 8     TMA producer: both Q tiles once, then K and V tiles of 128 keys
 //              (eight 16-token pages each, through the page table) into a
 //              two-stage ring
-//   warp 9     MMA issuer (tcgen05.mma, bf16 in, f32 accumulate in TMEM):
-//              S_A(0) S_B(0), then batches PV_A(j) S_A(j+1) | PV_B(j) S_B(j+1),
-//              in this order, so one tile's products run while the other
-//              tile's softmax works. The barriers a batch needs are waited on
-//              by different lanes at once.
+//   warps 9,10 MMA issuers of tile A and tile B (tcgen05.mma, bf16 in, f32
+//              accumulate in TMEM), taking turns: S_A(0) S_B(0), then batches
+//              PV_A(j) S_A(j+1) | PV_B(j) S_B(j+1), in this order, so one
+//              tile's products run while the other tile's softmax works. Each
+//              waits for its tile's P and the K / V stages (different lanes at
+//              once) while the other's batch is queued, and hands over two
+//              products before its own batch ends.
 //   warps 0-3  softmax of tile A, warps 4-7 softmax of tile B: thread i of a
 //              warpgroup owns TMEM lane i (= tile row i); online softmax in the
 //              log2 domain, the running max moved only past 2^8 growth (then O
@@ -44,9 +46,10 @@ constexpr int BM = 128;   // query rows per tile
 constexpr int BN = 128;   // keys per tile
 constexpr int D = kHeadDim;
 constexpr int kStages = 2;
-constexpr int kThreads = 320;
+constexpr int kThreads = 352;
 constexpr int kProducerWarp = 8;
-constexpr int kMmaWarp = 9;
+constexpr int kMmaWarp = 9;      // issues tile A's products (and owns TMEM)
+constexpr int kMmaWarpB = 10;    // issues tile B's products
 constexpr uint32_t kTileBytes = BM * D * 2;   // 32 KiB
 constexpr uint32_t kHalf = 16384;             // one 64-column half of a tile
 constexpr uint64_t kBudgetNs = 2000000000ull; // 2 s per wait
@@ -68,7 +71,10 @@ enum {
   B_OD = 13,     // +tile
   B_FIN = 15,
   B_VZ = 16,     // last V tile's rows past kv_len are zeroed
-  kNumBars = 17
+  B_HA = 17,     // tile A's issuer has issued its batch (tile B's may issue)
+  B_HB = 18,     // tile B's issuer has issued its batch
+  B_FIN2 = 19,
+  kNumBars = 20
 };
 constexpr uint32_t OFF_MISC = OFF_BAR + kNumBars * 8;
 constexpr uint32_t kSmemUsed = OFF_MISC + 16;
@@ -393,8 +399,8 @@ attention_kernel(const __grid_constant__ AttnLaunch p, const __grid_constant__ A
     for (int s = 0; s < kStages; ++s) {
       mbar_init(bar(B_KF + s), 1);
       mbar_init(bar(B_VF + s), 1);
-      mbar_init(bar(B_KE + s), 1);
-      mbar_init(bar(B_VE + s), 1);
+      mbar_init(bar(B_KE + s), n_q);   // one commit per issuing warp
+      mbar_init(bar(B_VE + s), n_q);
     }
     for (int x = 0; x < 2; ++x) {
       mbar_init(bar(B_SF + x), 1);
@@ -402,6 +408,9 @@ attention_kernel(const __grid_constant__ AttnLaunch p, const __grid_constant__ A
       mbar_init(bar(B_OD + x), 1);
     }
     mbar_init(bar(B_FIN), 1);
+    mbar_init(bar(B_FIN2), 1);
+    mbar_init(bar(B_HA), 1);
+    mbar_init(bar(B_HB), 1);
     mbar_init(bar(B_VZ), 1);
     *abort = 0;
     *never = 0;
@@ -496,7 +505,7 @@ attention_kernel(const __grid_constant__ AttnLaunch p, const __grid_constant__ A
           mbar_wait(bar(B_VF + (it & 1)), (it >> 1) & 1, kDrainNs, never);
       }
     }
-  } else if (warp == kMmaWarp) {
+  } else if (warp == kMmaWarp || warp == kMmaWarpB) {
     // ------------------------------------------------------ MMA issuer
     constexpr uint32_t idesc_qk = idesc_bf16_f32(BM, BN, false);
     const uint32_t idesc_pv = idesc_bf16_f32(BM, D, !vt);
@@ -531,14 +540,28 @@ attention_kernel(const __grid_constant__ AttnLaunch p, const __grid_constant__ A
       const bool wt = done || mbar_wait(br, par, kBudgetNs, abort, gabort);
       return __all_sync(0xffffffffu, wt);
     };
+    // Two issuing warps, one per query tile, in strict alternation: each waits
+    // for its own tile's P (and the K / V stages) and for the other's hand-off
+    // while the other's batch is queued, so the tensor pipe sees the single
+    // ordered stream PV_A S_A PV_B S_B ... with the waits taken off its path.
+    // (One warp issuing both tiles spent ~1200 cycles per batch on its commits,
+    // barrier polls and fence while the short product queue ran dry.) The
+    // hand-off orders only the issue: every product still waits for its own
+    // data through the barriers above.
+    const int x = warp == kMmaWarp ? 0 : 1;
     bool ok = true;
-    if (n_tiles > 0) {
-      ok = wait4(bar(B_Q), 0, bar(B_KF), 0, 0, 0, 0, 0);
+    if (n_tiles > 0 && x < n_q) {
+      const uint32_t t_s = tmem + TM_S + x * 128, t_o = tmem + TM_O + x * 128;
+      const uint64_t dq = x ? dq1 : dq0;
+      const uint32_t h_own = bar(x ? B_HB : B_HA), h_other = bar(x ? B_HA : B_HB);
+      const bool pair = n_q == 2;
+      // tile B's first S follows tile A's (hand-off phase 0)
+      ok = wait4(bar(B_Q), 0, bar(B_KF), 0, x ? h_other : 0u, 0, 0, 0);
       if (ok && lane == 0) {
         tc_fence_after();
-        for (int x = 0; x < n_q; ++x)
-          issue_s(tmem + TM_S + x * 128, x ? dq1 : dq0, dk0, idesc_qk, bar(B_SF + x));
+        issue_s(t_s, dq, dk0, idesc_qk, bar(B_SF + x));
         mma_commit(bar(B_KE + 0));
+        if (pair) mbar_arrive(h_own);
       }
       __syncwarp();
       for (int j = 0; ok && j < n_tiles; ++j) {
@@ -546,44 +569,53 @@ attention_kernel(const __grid_constant__ AttnLaunch p, const __grid_constant__ A
         const int nst = (j + 1) & 1;
         const bool more = j + 1 < n_tiles;
         const bool ragged = (w.kt_begin + j) * BN + BN > sq.kv_len;
-        for (int x = 0; ok && x < n_q; ++x) {
-          if (x == 0)
-            ok = wait4(bar(B_PF), j & 1, bar(B_VF + st), (j >> 1) & 1,
-                       more ? bar(B_KF + nst) : 0u, ((j + 1) >> 1) & 1, ragged ? bar(B_VZ) : 0u, 0);
-          else
-            ok = wait4(bar(B_PF + x), j & 1, 0, 0, 0, 0, 0, 0);
-          if (!ok) break;
-          if (lane == 0) {
-            tc_fence_after();
-            if constexpr (kShort) {
-              // short rows: key tile 0 also reads the remainder of P
-              if (short_rows && j == 0)
-                issue_pv_rem(tmem + TM_O + x * 128, tmem + TM_S + x * 128, st ? dv1 : dv0,
-                             v_step, idesc_pv);
-              else
-                issue_pv(tmem + TM_O + x * 128, tmem + TM_S + x * 128, st ? dv1 : dv0, v_step,
-                         idesc_pv, j == 0);
-            } else {
-              issue_pv(tmem + TM_O + x * 128, tmem + TM_S + x * 128, st ? dv1 : dv0, v_step,
-                       idesc_pv, j == 0);
-            }
-            if (x == n_q - 1) mma_commit(bar(B_VE + st));
-            if (more) {
-              issue_s(tmem + TM_S + x * 128, x ? dq1 : dq0, nst ? dk1 : dk0, idesc_qk,
-                      bar(B_SF + x));
-              if (x == n_q - 1) mma_commit(bar(B_KE + nst));
-            } else {
-              mma_commit(bar(B_OD + x));
-            }
+        // A's batch j follows B's batch j - 1 (B's hand-off phase j); B's batch j
+        // follows A's batch j (A's hand-off phase j + 1).
+        ok = wait4(bar(B_PF + x), j & 1, bar(B_VF + st), (j >> 1) & 1,
+                   more ? bar(B_KF + nst) : (ragged ? bar(B_VZ) : 0u), more ? ((j + 1) >> 1) & 1 : 0u,
+                   pair ? h_other : 0u, x ? (j + 1) & 1 : j & 1);
+        if (!ok) break;
+        if (lane == 0) {
+          tc_fence_after();
+          if constexpr (kShort) {
+            // short rows: key tile 0 also reads the remainder of P
+            if (short_rows && j == 0)
+              issue_pv_rem(t_o, t_s, st ? dv1 : dv0, v_step, idesc_pv);
+            else
+              issue_pv(t_o, t_s, st ? dv1 : dv0, v_step, idesc_pv, j == 0);
+          } else {
+            issue_pv(t_o, t_s, st ? dv1 : dv0, v_step, idesc_pv, j == 0);
           }
-          __syncwarp();
+          // The hand-off comes two products before the batch ends, so that the
+          // other issuer's wait ends as the queue runs out (c5 re-prefill per
+          // layer, by products left at the hand-off: 0 7.31 ms, 2 7.16-7.20,
+          // 4 7.17-7.23, 6 7.27, 8 7.51, 12 8.12); the commits follow it.
+          if (more) {
+            const uint64_t dk = nst ? dk1 : dk0;
+#pragma unroll
+            for (int kk = 0; kk < D / 16; ++kk) {
+              if (kk == D / 16 - 2 && pair) mbar_arrive(h_own);
+              const uint64_t o = static_cast<uint64_t>(((kk >> 2) * kHalf + (kk & 3) * 32) >> 4);
+              mma_bf16(t_s, dq + o, dk + o, idesc_qk, kk > 0 ? 1u : 0u);
+            }
+          } else if (pair) {
+            mbar_arrive(h_own);
+          }
+          mma_commit(bar(B_VE + st));
+          if (more) {
+            mma_commit(bar(B_SF + x));
+            mma_commit(bar(B_KE + nst));
+          } else {
+            mma_commit(bar(B_OD + x));
+          }
         }
+        __syncwarp();
       }
       if (!ok && lane == 0) record_timeout(abort);
       // Every MMA this thread issued has finished before TMEM is released.
-      if (lane == 0) mma_commit(bar(B_FIN));
+      if (lane == 0) mma_commit(bar(x ? B_FIN2 : B_FIN));
       __syncwarp();
-      mbar_wait(bar(B_FIN), 0, kDrainNs, never);
+      mbar_wait(bar(x ? B_FIN2 : B_FIN), 0, kDrainNs, never);
     }
   } else {
     // ------------------------------------------------------ softmax warpgroups
