@@ -359,16 +359,18 @@ nexus_status plan_attention(int32_t n_seqs, const int32_t* kv_len, const int32_t
     }
     pl.splits = pl.splits_pair = pl.splits_single = best;
     // Split, all CTAs in one wave, pairs of both kinds present: a pair holding
-    // one query tile runs a key-tile step in ~0.87 of a two-tile pair's time and
-    // ends ~3 steps sooner (one tile to write back), so it takes fewer splits
-    // over longer key ranges and the two kinds end together. Measured on the c5
-    // suffix (9 splits each): two-tile pairs end at ~63 us, one-tile pairs at ~52.
+    // one query tile runs a key-tile step in about a two-tile pair's time (whose
+    // two issuing warps take turns; a one-tile pair has one) and ends ~3 steps
+    // sooner (one tile to write back), so the two kinds take their own split
+    // counts and end together. Calibrated on the c5 suffix, swept over the
+    // counts (two-tile / one-tile pairs, one layer): 10 / 9 57.4 us, 9 / 9 58.6,
+    // 11 / 8 60.8, 10 / 8 60.5, 9 / 10 62.1, 8 / 8 63.2.
     const int64_t units = static_cast<int64_t>(n_kv_heads) * std::max(1, n_layers_call);
     bool short_rows = false;   // tile pairs whose rows see fewer than 128 keys: uniform splits
     for (int32_t s = 0; s < n_seqs; ++s)
       short_rows = short_rows || (q_len[s] > 0 && kv_len[s] - q_len[s] < 127);
     if (best > 1 && n_pair > 0 && n_single > 0 && ctas * best <= sms && !short_rows) {
-      constexpr double kSingleStep = 0.87, kPairFixed = 6.1, kSingleFixed = 3.2;
+      constexpr double kSingleStep = 1.0, kPairFixed = 6.1, kSingleFixed = 3.2;
       auto span = [&](int sp, int ss) {
         const double tp = std::ceil(static_cast<double>(kt_pair) / sp) + kPairFixed;
         const double ts = kSingleStep * std::ceil(static_cast<double>(kt_single) / ss) + kSingleFixed;
