@@ -192,8 +192,11 @@ qkv_kernel(const __grid_constant__ QkvLaunch p, const __grid_constant__ QkvMaps 
   if constexpr (kPair) cluster_sync_all();
   const uint32_t tmem = *tmem_slot;
   // Launched with programmatic stream serialization: the setup above overlaps
-  // the previous kernel's tail; no global memory is touched before it ends.
-  griddep_wait();
+  // the previous kernel's tail, and no global memory this or an earlier kernel
+  // writes is touched before that kernel has ended. The one exception is the
+  // producer's first weight rows: the weights are read-only to every kernel of
+  // this library, so they are requested before the wait.
+  if (warp != kProducerWarp) griddep_wait();
   griddep_launch_dependents();
 
   if (warp == kProducerWarp) {
@@ -204,6 +207,24 @@ qkv_kernel(const __grid_constant__ QkvLaunch p, const __grid_constant__ QkvMaps 
       // Every band of token tiles reads the whole weight again: it is kept in L2
       // ahead of the activation rows and the outputs streaming past it.
       const uint64_t w_policy = l2_policy_evict_last();
+      // the first tile's first stages: weight rows now (each stage's full
+      // barrier expects its whole bytes), activation rows after the wait
+      int n_pre = 0;
+      if (t_first < p.total_tiles) {
+        int mt, nt;
+        tile_coords(p, t_first, mt, nt);
+        n_pre = min(kStages, kb1 - kb0);
+        for (int st = 0; st < n_pre; ++st) {
+          const int kb = kb0 + st;
+          const uint32_t a = sbase + st * kStageBytes;
+          mbar_arrive_expect_tx(bar(B_FULL + st), kStageBytes);
+#pragma unroll
+          for (int sub = 0; sub < kSub; ++sub)
+            tma_load_2d_hint(a + sub * kSubBytes + kABytes, &maps.w, bar(B_FULL + st),
+                             (kb * kSub + sub) * BK, nt * BN, w_policy);
+        }
+      }
+      griddep_wait();
       int it = 0;
       bool ok = true;
       for (int t = t_first; t < p.total_tiles && ok; t += t_step) {
@@ -216,12 +237,14 @@ qkv_kernel(const __grid_constant__ QkvLaunch p, const __grid_constant__ QkvMaps 
             if (!ok) { record_timeout(abort); break; }
           }
           const uint32_t a = sbase + st * kStageBytes;
-          mbar_arrive_expect_tx(bar(B_FULL + st), kStageBytes);
+          const bool pre = it < n_pre;   // weight rows already requested
+          if (!pre) mbar_arrive_expect_tx(bar(B_FULL + st), kStageBytes);
 #pragma unroll
           for (int sub = 0; sub < kSub; ++sub) {
             tma_load_2d(a + sub * kSubBytes, &maps.x, bar(B_FULL + st), (kb * kSub + sub) * BK, mt * BM);
-            tma_load_2d_hint(a + sub * kSubBytes + kABytes, &maps.w, bar(B_FULL + st),
-                             (kb * kSub + sub) * BK, nt * BN, w_policy);
+            if (!pre)
+              tma_load_2d_hint(a + sub * kSubBytes + kABytes, &maps.w, bar(B_FULL + st),
+                               (kb * kSub + sub) * BK, nt * BN, w_policy);
           }
         }
       }
