@@ -442,6 +442,8 @@ attention_kernel(const __grid_constant__ AttnLaunch p, const __grid_constant__ A
         prefetch_tmap(&maps.q);
         prefetch_tmap(&maps.k);
         prefetch_tmap(&maps.v);
+        prefetch_tmap(&maps.k8);
+        prefetch_tmap(&maps.v8);
         mbar_arrive_expect_tx(bar(B_Q), 2u * n_q * G * p.tile_tokens * 128u);
         for (int x = 0; x < n_q; ++x)
           for (int half = 0; half < 2; ++half)
@@ -457,13 +459,24 @@ attention_kernel(const __grid_constant__ AttnLaunch p, const __grid_constant__ A
         int page = 0;
         if (lane < 8) page = pt[min(kt * 8 + lane, pg_max)];
         const int gp = layer * p.n_pages + page;
+        // Eight consecutive page ids (the clamped ids of a ragged last tile
+        // repeat, so it never qualifies): each 64-column half of the tile is one
+        // copy of eight pages, which lands in the same rows as eight copies.
+        const int gp0 = __shfl_sync(0xffffffffu, gp, 0);
+        const bool run8 = __all_sync(0xffffffffu, lane >= 8 || gp == gp0 + lane);
         bool ok = true;
         if (it >= 2) ok = mbar_wait(bar(B_KE + st), ((it >> 1) - 1) & 1, kBudgetNs, abort, gabort);
         ok = __all_sync(0xffffffffu, ok);
         if (!ok) { if (lane == 0) record_timeout(abort); break; }
         if (lane == 0) mbar_arrive_expect_tx(bar(B_KF + st), kTileBytes);
         __syncwarp();
-        if (lane < 8) {
+        if (run8) {
+          if (lane == 0) {
+            const uint32_t kdst = sbase + OFF_K + st * kTileBytes;
+            tma_load_4d(kdst, &maps.k8, bar(B_KF + st), 0, 0, w.kv, gp0);
+            tma_load_4d(kdst + kHalf, &maps.k8, bar(B_KF + st), 64, 0, w.kv, gp0);
+          }
+        } else if (lane < 8) {
           const uint32_t kdst = sbase + OFF_K + st * kTileBytes + lane * 2048;
           tma_load_4d(kdst, &maps.k, bar(B_KF + st), 0, 0, w.kv, gp);
           tma_load_4d(kdst + kHalf, &maps.k, bar(B_KF + st), 64, 0, w.kv, gp);
@@ -473,7 +486,17 @@ attention_kernel(const __grid_constant__ AttnLaunch p, const __grid_constant__ A
         if (!ok) { if (lane == 0) record_timeout(abort); issued_k = it + 1; break; }
         if (lane == 0) mbar_arrive_expect_tx(bar(B_VF + st), kTileBytes);
         __syncwarp();
-        if (lane < 8) {
+        if (run8) {
+          if (lane == 0) {
+            const uint32_t vdst = sbase + OFF_V + st * kTileBytes;
+            if (!vt) {
+              tma_load_4d(vdst, &maps.v8, bar(B_VF + st), 0, 0, w.kv, gp0);
+              tma_load_4d(vdst + kHalf, &maps.v8, bar(B_VF + st), 64, 0, w.kv, gp0);
+            } else {
+              tma_load_4d(vdst, &maps.v8, bar(B_VF + st), 0, 0, w.kv, gp0);
+            }
+          }
+        } else if (lane < 8) {
           const uint32_t vdst = sbase + OFF_V + st * kTileBytes;
           if (!vt) {
             tma_load_4d(vdst + lane * 2048, &maps.v, bar(B_VF + st), 0, 0, w.kv, gp);

@@ -123,6 +123,10 @@ struct AttnMaps {
   CUtensorMap q;
   CUtensorMap k;
   CUtensorMap v;
+  // The same K / V with boxes of eight pages: one copy per 64-column half of a
+  // key tile whose eight page ids are consecutive.
+  CUtensorMap k8;
+  CUtensorMap v8;
 };
 
 cudaError_t launch_attention(const AttnLaunch& p, const AttnMaps& maps, cudaStream_t stream);

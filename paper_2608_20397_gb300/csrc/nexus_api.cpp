@@ -529,10 +529,13 @@ nexus_status attention_impl(const nexus_kv_cache* c, const int32_t* d_pt, int32_
     const uint64_t dims[4] = {kHeadDim, kPageSize, static_cast<uint64_t>(c->n_kv_heads), gpages};
     const uint64_t strides[3] = {kHeadDim * 2, head_bytes, head_bytes * c->n_kv_heads};
     const uint32_t box[4] = {64, kPageSize, 1, 1};
-    if (!encode_4d(&maps.k, c->k_pool, dims, strides, box, CU_TENSOR_MAP_SWIZZLE_128B))
+    const uint32_t box8[4] = {64, kPageSize, 1, 8};   // eight consecutive pages
+    if (!encode_4d(&maps.k, c->k_pool, dims, strides, box, CU_TENSOR_MAP_SWIZZLE_128B) ||
+        !encode_4d(&maps.k8, c->k_pool, dims, strides, box8, CU_TENSOR_MAP_SWIZZLE_128B))
       return NEXUS_ECUDA;
     if (!c->v_transposed) {
-      if (!encode_4d(&maps.v, c->v_pool, dims, strides, box, CU_TENSOR_MAP_SWIZZLE_128B))
+      if (!encode_4d(&maps.v, c->v_pool, dims, strides, box, CU_TENSOR_MAP_SWIZZLE_128B) ||
+          !encode_4d(&maps.v8, c->v_pool, dims, strides, box8, CU_TENSOR_MAP_SWIZZLE_128B))
         return NEXUS_ECUDA;
     }
   }
@@ -540,7 +543,9 @@ nexus_status attention_impl(const nexus_kv_cache* c, const int32_t* d_pt, int32_
     const uint64_t dims[4] = {kPageSize, kHeadDim, static_cast<uint64_t>(c->n_kv_heads), gpages};
     const uint64_t strides[3] = {kPageSize * 2, head_bytes, head_bytes * c->n_kv_heads};
     const uint32_t box[4] = {kPageSize, kHeadDim, 1, 1};
-    if (!encode_4d(&maps.v, c->v_pool, dims, strides, box, CU_TENSOR_MAP_SWIZZLE_32B))
+    const uint32_t box8[4] = {kPageSize, kHeadDim, 1, 8};
+    if (!encode_4d(&maps.v, c->v_pool, dims, strides, box, CU_TENSOR_MAP_SWIZZLE_32B) ||
+        !encode_4d(&maps.v8, c->v_pool, dims, strides, box8, CU_TENSOR_MAP_SWIZZLE_32B))
       return NEXUS_ECUDA;
   }
   if (launch_attention(*p, maps, stream) != cudaSuccess) return NEXUS_ECUDA;

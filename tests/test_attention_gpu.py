@@ -15,15 +15,18 @@ DEV = torch.device("cuda:0") if torch.cuda.is_available() else None
 
 
 def _direct_case(kv_lens, q_lens, Hq=40, H=8, L=1, vt=False, seed=0, shuffle=True,
-                 garbage=True, vscale=1.0):
+                 garbage=True, vscale=1.0, order=None):
     """Sequences written straight into a paged pool (no splice); slots past
     kv_len hold NaN so any leak of them into the output shows. vscale (a power
-    of two, so exact in bf16) scales V."""
+    of two, so exact in bf16) scales V. `order` (a permutation of the pool's
+    pages) overrides `shuffle`."""
     rng = np.random.default_rng(seed)
     max_pages = max(-(-k // 16) for k in kv_lens) + 1
     n_pages = sum(-(-k // 16) for k in kv_lens) + 8
     kp, vp = new_pools(L, n_pages, H, vt, DEV, float("nan") if garbage else 0.0)
-    order = rng.permutation(n_pages) if shuffle else np.arange(n_pages)
+    if order is None:
+        order = rng.permutation(n_pages) if shuffle else np.arange(n_pages)
+    assert sorted(order) == list(range(n_pages))
     h_pt = np.full((len(kv_lens), max_pages), -1, np.int32)
     ks, vs, cur = [], [], 0
     for i, T in enumerate(kv_lens):
@@ -164,6 +167,39 @@ def test_split_kv_one_tile_pair_both_slots(kv, ql, split, vt, cap):
                                        softcap=cap)
         assert nexus.device_status() == nexus.OK
     _check(ks, vs, q, o, lse, kv, ql, 5, what=f"one-tile pair split {split}", softcap=cap)
+
+
+def _runs_of_eight(n_pages, offset, seed):
+    """Pages in runs of eight consecutive ids, the runs shuffled, the whole
+    order rotated by `offset` so runs start off key-tile boundaries."""
+    rng = np.random.default_rng(seed)
+    runs = [list(range(i, min(i + 8, n_pages))) for i in range(0, n_pages, 8)]
+    rng.shuffle(runs)
+    order = [p for r in runs for p in r]
+    return np.array(order[offset:] + order[:offset])
+
+
+# A key tile whose eight page ids are consecutive is copied with one box per
+# 64-column half (eight pages each); others page by page. Pages in order (every
+# full tile takes the eight-page copies), and runs of eight shuffled and rotated
+# (tiles of both kinds, runs starting inside a tile); both V layouts, split and
+# unsplit plans, a ragged last tile.
+@pytest.mark.parametrize("vt,split,layout", [
+    (False, 1, "in order"), (True, 1, "in order"), (False, 4, "in order"), (True, 0, "in order"),
+    (False, 1, "runs"), (True, 3, "runs"), (False, 0, "runs+3")])
+def test_contiguous_page_runs(vt, split, layout):
+    kv, ql = [3001, 1500], [300, 64]
+    n_pages = sum(-(-k // 16) for k in kv) + 8
+    order = None
+    if layout == "in order":
+        order = np.arange(n_pages)
+    elif layout == "runs":
+        order = _runs_of_eight(n_pages, 0, 5)
+    else:
+        order = _runs_of_eight(n_pages, 3, 6)
+    cache, d_pt, mp, ks, vs, q = _direct_case(kv, ql, vt=vt, seed=31 + split, order=order)
+    o, lse = _run(cache, d_pt, mp, kv, ql, q, 40, 1, split_kv=split)
+    _check(ks, vs, q, o, lse, kv, ql, 5, what=f"pages {layout} split {split} vt {vt}")
 
 
 def test_reprefill_equals_textbook_causal():
