@@ -9,7 +9,8 @@
 //
 //   warp 8     TMA producer: both Q tiles once, then K and V tiles of 128 keys
 //              (eight 16-token pages each, through the page table) into a
-//              two-stage ring
+//              two-stage ring; a tile whose eight page ids are consecutive is
+//              one copy per 64-column half, any other one copy per page and half
 //   warps 9,10 MMA issuers of tile A and tile B (tcgen05.mma, bf16 in, f32
 //              accumulate in TMEM), taking turns: S_A(0) S_B(0), then batches
 //              PV_A(j) S_A(j+1) | PV_B(j) S_B(j+1), in this order, so one
