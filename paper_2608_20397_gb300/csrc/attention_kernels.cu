@@ -1008,12 +1008,13 @@ cudaError_t launch_attention(const AttnLaunch& p, const AttnMaps& maps, cudaStre
   if (p.total_tiles <= 0 || p.n_layers_call <= 0) return cudaSuccess;
   static_assert(kSmemBytes <= 227 * 1024, "shared memory budget");
   const bool kinds = p.splits > 1 && !p.short_rows && p.cta_prefix[p.n_seqs] > 0;
+  // (short-row launches never take a kinds plan)
   void (*kernel)(const AttnLaunch, const AttnMaps);
   if (p.softcap_out > 0.f)
-    kernel = p.short_rows ? (kinds ? attention_kernel<true, true, true> : attention_kernel<true, true, false>)
+    kernel = p.short_rows ? attention_kernel<true, true, false>
                           : (kinds ? attention_kernel<true, false, true> : attention_kernel<true, false, false>);
   else
-    kernel = p.short_rows ? (kinds ? attention_kernel<false, true, true> : attention_kernel<false, true, false>)
+    kernel = p.short_rows ? attention_kernel<false, true, false>
                           : (kinds ? attention_kernel<false, false, true> : attention_kernel<false, false, false>);
   cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        (int)kSmemBytes);
