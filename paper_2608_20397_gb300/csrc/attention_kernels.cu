@@ -15,14 +15,17 @@
 //              accumulate in TMEM), taking turns: S_A(0) S_B(0), then batches
 //              PV_A(j) S_A(j+1) | PV_B(j) S_B(j+1), in this order, so one
 //              tile's products run while the other tile's softmax works. Each
-//              waits for its tile's P and the K / V stages (different lanes at
-//              once) while the other's batch is queued, and hands over two
-//              products before its own batch ends.
+//              waits for its tile's P of the first 80 keys and the K / V stages
+//              (different lanes at once) while the other's batch is queued,
+//              queues those keys' P V products, checks that the rest of P has
+//              landed, and hands over two products before its own batch ends.
 //   warps 0-3  softmax of tile A, warps 4-7 softmax of tile B: thread i of a
 //              warpgroup owns TMEM lane i (= tile row i); online softmax in the
 //              log2 domain, the running max moved only past 2^8 growth (then O
 //              is rescaled in TMEM); P is written back as bf16 over the first 64
-//              columns of the tile's own S and read from TMEM by the P V product
+//              columns of the tile's own S, in two parts (keys 0-79, then
+//              80-127, each released by its own barrier), and read from TMEM by
+//              the P V product
 //
 // TMEM columns: S_A [0,128), S_B [128,256), O_A [256,384), O_B [384,512).
 // The S-full barrier of tile X at step j is committed after PV_X(j-1), so it
@@ -32,6 +35,7 @@
 #include <cuda_bf16.h>
 
 #include <mutex>
+#include <type_traits>
 
 #include "internal.h"
 #include "ptx.cuh"
@@ -56,6 +60,9 @@ constexpr uint32_t kHalf = 16384;             // one 64-column half of a tile
 constexpr uint64_t kBudgetNs = 2000000000ull; // 2 s per wait
 constexpr uint64_t kDrainNs = 200000000ull;   // 0.2 s to drain after an abort
 constexpr float kRescaleThreshold = 8.0f;     // move the running max only past 2^8 growth
+// The softmax releases P of a tile's first kLoKeys keys before the rest, so the
+// issuer wakes and queues those P V products while the rest of P is computed.
+constexpr int kLoKeys = 80;
 
 constexpr uint32_t OFF_Q = 0;                          // tile A, tile B
 constexpr uint32_t OFF_K = OFF_Q + 2 * kTileBytes;
@@ -68,14 +75,16 @@ enum {
   B_KE = 5,      // +stage: K tile consumed (every tile's S product done)
   B_VE = 7,      // +stage: V tile consumed (every tile's P V product done)
   B_SF = 9,      // +tile
-  B_PF = 11,     // +tile
+  B_PF = 11,     // +tile: P of keys [0, kLoKeys) stored
   B_OD = 13,     // +tile
   B_FIN = 15,
   B_VZ = 16,     // last V tile's rows past kv_len are zeroed
   B_HA = 17,     // tile A's issuer has issued its batch (tile B's may issue)
   B_HB = 18,     // tile B's issuer has issued its batch
   B_FIN2 = 19,
-  kNumBars = 20
+  B_PH = 20,     // +tile: P of keys [kLoKeys, 128) stored
+  B_PL = 22,     // +tile: the P V products of keys [0, kLoKeys) are done
+  kNumBars = 24
 };
 constexpr uint32_t OFF_MISC = OFF_BAR + kNumBars * 8;
 constexpr uint32_t kSmemUsed = OFF_MISC + 16;
@@ -328,11 +337,13 @@ __device__ __forceinline__ void issue_s(uint32_t t_s, uint64_t dq, uint64_t dk, 
   mma_commit(s_full);
 }
 
-// O += P V over one 128-key tile: P from TMEM (16 keys = 8 columns per step).
+// O += P V over keys [16 kk0, 16 kk1) of a 128-key tile: P from TMEM (16 keys
+// = 8 columns per step).
+template <int kk0, int kk1>
 __device__ __forceinline__ void issue_pv(uint32_t t_o, uint32_t t_s, uint64_t dv, uint64_t v_step,
                                          uint32_t idesc, bool first) {
 #pragma unroll
-  for (int kk = 0; kk < BN / 16; ++kk)
+  for (int kk = kk0; kk < kk1; ++kk)
     mma_bf16_ts(t_o, t_s + kk * 8, dv + kk * v_step, idesc, (!first || kk > 0) ? 1u : 0u);
 }
 
@@ -406,6 +417,8 @@ attention_kernel(const __grid_constant__ AttnLaunch p, const __grid_constant__ A
     for (int x = 0; x < 2; ++x) {
       mbar_init(bar(B_SF + x), 1);
       mbar_init(bar(B_PF + x), 128);
+      mbar_init(bar(B_PH + x), 128);
+      mbar_init(bar(B_PL + x), 1);
       mbar_init(bar(B_OD + x), 1);
     }
     mbar_init(bar(B_FIN), 1);
@@ -599,17 +612,28 @@ attention_kernel(const __grid_constant__ AttnLaunch p, const __grid_constant__ A
                    more ? bar(B_KF + nst) : (ragged ? bar(B_VZ) : 0u), more ? ((j + 1) >> 1) & 1 : 0u,
                    pair ? h_other : 0u, x ? (j + 1) & 1 : j & 1);
         if (!ok) break;
+        // short rows: key tile 0 also reads the remainder of P, all after the
+        // whole of P (the softmax releases both parts at once there)
+        bool rem0 = false;
+        if constexpr (kShort) rem0 = short_rows && j == 0;
+        const uint64_t dv = st ? dv1 : dv0;
+        bool got = true;
         if (lane == 0) {
           tc_fence_after();
-          if constexpr (kShort) {
-            // short rows: key tile 0 also reads the remainder of P
-            if (short_rows && j == 0)
-              issue_pv_rem(t_o, t_s, st ? dv1 : dv0, v_step, idesc_pv);
-            else
-              issue_pv(t_o, t_s, st ? dv1 : dv0, v_step, idesc_pv, j == 0);
-          } else {
-            issue_pv(t_o, t_s, st ? dv1 : dv0, v_step, idesc_pv, j == 0);
-          }
+          if (!rem0) issue_pv<0, kLoKeys / 16>(t_o, t_s, dv, v_step, idesc_pv, j == 0);
+          mma_commit(bar(B_PL + x));
+          // The rest of P has usually landed while those products were queued:
+          // the issuing thread checks in place (a warp-wide wait here stalled
+          // the product stream for ~200 cycles and drained the queue).
+          got = mbar_test_wait(bar(B_PH + x), j & 1) ||
+                mbar_wait(bar(B_PH + x), j & 1, kBudgetNs, abort, gabort);
+        }
+        if (lane == 0 && got) {
+          tc_fence_after();
+          if (rem0)
+            issue_pv_rem(t_o, t_s, dv, v_step, idesc_pv);
+          else
+            issue_pv<kLoKeys / 16, BN / 16>(t_o, t_s, dv, v_step, idesc_pv, false);
           // The hand-off comes two products before the batch ends, so that the
           // other issuer's wait ends as the queue runs out (c5 re-prefill per
           // layer, by products left at the hand-off: 0 7.31 ms, 2 7.16-7.20,
@@ -633,7 +657,7 @@ attention_kernel(const __grid_constant__ AttnLaunch p, const __grid_constant__ A
             mma_commit(bar(B_OD + x));
           }
         }
-        __syncwarp();
+        ok = __shfl_sync(0xffffffffu, got ? 1 : 0, 0) != 0;
       }
       if (!ok && lane == 0) record_timeout(abort);
       // Every MMA this thread issued has finished before TMEM is released.
@@ -675,52 +699,57 @@ attention_kernel(const __grid_constant__ AttnLaunch p, const __grid_constant__ A
 #pragma unroll
           for (int e = 0; e < 32; ++e) s[q * 32 + e] = __uint_as_float(v[q][e]);
       }
-      if constexpr (kSoftcap) {
-        // tanh(x) = 2 / (2 z) - 1 with 2 z = 1 + u, u = 2^(-2 x log2 e); the
-        // argument is clamped at 30 so that u stays finite (and a NaN score of an
-        // unused slot, masked below, becomes a finite number). The reciprocals of a
-        // group of four z come from one: 1 / z_i = (product of the other three) /
-        // (product of all four).
-        const float2 nci = make_float2(-p.softcap_in, -p.softcap_in);
-        const float2 half = make_float2(0.5f, 0.5f), mone = make_float2(-1.f, -1.f);
-#pragma unroll
-        for (int c = 0; c < BN; c += 4) {
-          float2 a = fmul2(make_float2(s[c], s[c + 1]), nci);
-          float2 b = fmul2(make_float2(s[c + 2], s[c + 3]), nci);
-          a.x = ex2_approx(fminf(a.x, 30.f));
-          a.y = ex2_approx(fminf(a.y, 30.f));
-          b.x = ex2_approx(fminf(b.x, 30.f));
-          b.y = ex2_approx(fminf(b.y, 30.f));
-          const float2 za = ffma2(a, half, half);
-          const float2 zb = ffma2(b, half, half);
-          const float2 zp = fmul2(za, zb);
-          const float r = rcp_approx(zp.x * zp.y);
-          const float2 rp = fmul2(make_float2(r, r), make_float2(zp.y, zp.x));
-          const float2 ta = ffma2(rp, zb, mone);
-          const float2 tb = ffma2(rp, za, mone);
-          s[c] = ta.x;
-          s[c + 1] = ta.y;
-          s[c + 2] = tb.x;
-          s[c + 3] = tb.y;
-        }
-      }
       const int lim = pos_r - (w.kt_begin + j) * BN;   // keys c <= lim are visible
-      if (lim < BN - 1) {
+      // Columns [c0, c1) made ready for the exponentials: soft-capped, then
+      // masked. The row is prepared in two parts, [0, kLoKeys) first.
+      auto prep = [&](auto c0c, auto c1c) {
+        constexpr int c0 = decltype(c0c)::value, c1 = decltype(c1c)::value;
+        if constexpr (kSoftcap) {
+          // tanh(x) = 2 / (2 z) - 1 with 2 z = 1 + u, u = 2^(-2 x log2 e); the
+          // argument is clamped at 30 so that u stays finite (and a NaN score of
+          // an unused slot, masked below, becomes a finite number). The
+          // reciprocals of a group of four z come from one: 1 / z_i = (product
+          // of the other three) / (product of all four).
+          const float2 nci = make_float2(-p.softcap_in, -p.softcap_in);
+          const float2 half = make_float2(0.5f, 0.5f), mone = make_float2(-1.f, -1.f);
 #pragma unroll
-        for (int c = 0; c < BN; ++c) s[c] = (c <= lim) ? s[c] : -INFINITY;
-      }
-      // One pass over the row: exponentials 2^(s sc - m) written to TMEM as
-      // bf16 P over the first 64 columns of S, and four pair chains of the row
-      // sum.
+          for (int c = c0; c < c1; c += 4) {
+            float2 a = fmul2(make_float2(s[c], s[c + 1]), nci);
+            float2 b = fmul2(make_float2(s[c + 2], s[c + 3]), nci);
+            a.x = ex2_approx(fminf(a.x, 30.f));
+            a.y = ex2_approx(fminf(a.y, 30.f));
+            b.x = ex2_approx(fminf(b.x, 30.f));
+            b.y = ex2_approx(fminf(b.y, 30.f));
+            const float2 za = ffma2(a, half, half);
+            const float2 zb = ffma2(b, half, half);
+            const float2 zp = fmul2(za, zb);
+            const float r = rcp_approx(zp.x * zp.y);
+            const float2 rp = fmul2(make_float2(r, r), make_float2(zp.y, zp.x));
+            const float2 ta = ffma2(rp, zb, mone);
+            const float2 tb = ffma2(rp, za, mone);
+            s[c] = ta.x;
+            s[c + 1] = ta.y;
+            s[c + 2] = tb.x;
+            s[c + 3] = tb.y;
+          }
+        }
+        if (lim < c1 - 1) {
+#pragma unroll
+          for (int c = c0; c < c1; ++c) s[c] = (c <= lim) ? s[c] : -INFINITY;
+        }
+      };
+      // Exponentials 2^(s sc - m) of columns [16 q0, 16 q1), written to TMEM as
+      // bf16 P over the first 64 columns of S; returns their row sum (four pair
+      // chains).
       float2 sum[4];
-      float mxa[8];
-      auto pass = [&](float neg_m) {
+      auto pass = [&](auto q0c, auto q1c, float neg_m) -> float {
+        constexpr int q0 = decltype(q0c)::value, q1 = decltype(q1c)::value;
         const float2 sc2 = make_float2(sc, sc);
         const float2 nm2 = make_float2(neg_m, neg_m);
 #pragma unroll
         for (int k = 0; k < 4; ++k) sum[k] = make_float2(0.f, 0.f);
 #pragma unroll
-        for (int q = 0; q < 8; ++q) {
+        for (int q = q0; q < q1; ++q) {
           uint32_t pk[8];
 #pragma unroll
           for (int e = 0; e < 16; e += 2) {
@@ -733,11 +762,14 @@ attention_kernel(const __grid_constant__ AttnLaunch p, const __grid_constant__ A
           }
           tmem_st8(t_s + q * 8, pk);   // P over the first 64 columns of S
         }
+        return ((sum[0].x + sum[0].y) + (sum[1].x + sum[1].y)) +
+               ((sum[2].x + sum[2].y) + (sum[3].x + sum[3].y));
       };
-      // The same pass for short rows' key tile 0, which also writes the bf16
-      // remainder P - bf16(P) over columns 64..127, four columns of each at a
-      // time (the score row already holds 128 of the thread's registers).
-      auto pass_rem = [&](float neg_m) {
+      // The same pass over the whole row for short rows' key tile 0, which also
+      // writes the bf16 remainder P - bf16(P) over columns 64..127, four columns
+      // of each at a time (the score row already holds 128 of the thread's
+      // registers).
+      auto pass_rem = [&](float neg_m) -> float {
         const float2 sc2 = make_float2(sc, sc);
         const float2 nm2 = make_float2(neg_m, neg_m);
 #pragma unroll
@@ -760,68 +792,117 @@ attention_kernel(const __grid_constant__ AttnLaunch p, const __grid_constant__ A
           tmem_st4(t_s + q * 4, pk);
           tmem_st4(t_s + BN / 2 + q * 4, pl);
         }
+        return ((sum[0].x + sum[0].y) + (sum[1].x + sum[1].y)) +
+               ((sum[2].x + sum[2].y) + (sum[3].x + sum[3].y));
       };
-      auto row_max = [&]() -> float {
+      // max over columns [c0, 128)
+      auto row_max = [&](auto c0c) -> float {
+        constexpr int c0 = decltype(c0c)::value;
+        float mxa[8];
+#pragma unroll
+        for (int k = 0; k < 8; ++k) mxa[k] = -INFINITY;
+#pragma unroll
+        for (int c = c0; c < BN; c += 16)
+#pragma unroll
+          for (int k = 0; k < 8; ++k) mxa[k] = fmax3(mxa[k], s[c + k], s[c + 8 + k]);
         return fmaxf(fmax3(mxa[0], mxa[1], mxa[2]),
                      fmaxf(fmax3(mxa[3], mxa[4], mxa[5]), fmaxf(mxa[6], mxa[7])));
       };
+      // O of this tile's rows scaled by alpha (warps whose rows all keep their
+      // max skip it).
+      auto rescale_o = [&](float alpha) {
+#pragma unroll 1
+        for (int q = 0; q < 4; ++q) {
+          uint32_t v[32];
+          tmem_ld32(t_o + q * 32, v);
+          tmem_ld_wait();
 #pragma unroll
-      for (int k = 0; k < 8; ++k) mxa[k] = -INFINITY;
+          for (int e = 0; e < 32; ++e) v[e] = __float_as_uint(__uint_as_float(v[e]) * alpha);
+          tmem_st32(t_o + q * 32, v);
+        }
+      };
       // The running max moves only when a tile's max exceeds it by more than
       // 2^8, which after a row's first tile is rare. So once every row of the
       // warp has a running max, the exponentials are taken with it straight
-      // away: if none of them exceeds 2^8 the max would not have moved, and a
-      // row sum below 2^8 proves that. A row whose sum reaches 2^8 (or is not
-      // a number) is redone with the max taken first, so the result is always
-      // that of taking the max first.
+      // away, part by part: a part's sum below 2^8 proves that none of its
+      // exponentials exceeds 2^8, i.e. the max would not have moved for them.
+      // P of keys [0, kLoKeys) is released as soon as that holds for them, and
+      // the issuer queues their P V products while the rest is computed. If the
+      // rest moves the max (its own max is then the row's), the softmax waits
+      // for those products, scales O (which then holds them) like any moved max
+      // does, and redoes the rest of P with the new max; a row whose first part
+      // already moves it (and every row's first tile) takes the max over the
+      // whole row first.
+      prep(std::integral_constant<int, 0>{}, std::integral_constant<int, kLoKeys>{});
       const bool have_max = __all_sync(0xffffffffu, m_run != -INFINITY);
-      bool check = true;
+      bool fast = false;
+      float rs_lo = 0.f;
       if (have_max) {
-        pass(-m_run);   // never short rows' key tile 0: no running max yet there
-        const float rowsum = ((sum[0].x + sum[0].y) + (sum[1].x + sum[1].y)) +
-                             ((sum[2].x + sum[2].y) + (sum[3].x + sum[3].y));
-        check = !(rowsum < 256.f);
+        rs_lo = pass(std::integral_constant<int, 0>{}, std::integral_constant<int, kLoKeys / 16>{},
+                     -m_run);
+        fast = !__any_sync(0xffffffffu, !(rs_lo < 256.f));
       }
-      float alpha = 1.f;
-      if (__any_sync(0xffffffffu, check)) {
-#pragma unroll
-        for (int c = 0; c < BN; c += 16)
-#pragma unroll
-          for (int k = 0; k < 8; ++k) mxa[k] = fmax3(mxa[k], s[c + k], s[c + 8 + k]);
-      }
-      const float mx = row_max();
-      const float mxs = mx * sc;
-      const bool move = mx > -INFINITY && (m_run == -INFINITY || mxs > m_run + kRescaleThreshold);
-      if (__any_sync(0xffffffffu, move || !have_max)) {
-        bool rescale = false;
-        if (move) {
-          if (m_run != -INFINITY) { alpha = ex2_approx(m_run - mxs); rescale = true; }
-          m_run = mxs;
-        }
-        if constexpr (kShort) {
-          if (short_rows && j == 0) pass_rem(m_run == -INFINITY ? 0.f : -m_run);
-          else pass(m_run == -INFINITY ? 0.f : -m_run);
-        } else {
-          pass(m_run == -INFINITY ? 0.f : -m_run);
-        }
-        if (__any_sync(0xffffffffu, rescale)) {
-          // PV_x(j-1) is complete: this step's S-full barrier was committed after it.
-#pragma unroll 1
-          for (int q = 0; q < 4; ++q) {
-            uint32_t v[32];
-            tmem_ld32(t_o + q * 32, v);
-            tmem_ld_wait();
-#pragma unroll
-            for (int e = 0; e < 32; ++e) v[e] = __float_as_uint(__uint_as_float(v[e]) * alpha);
-            tmem_st32(t_o + q * 32, v);
+      if (fast) {
+        tmem_st_wait();
+        tc_fence_before();
+        mbar_arrive(bar(B_PF + x));
+        prep(std::integral_constant<int, kLoKeys>{}, std::integral_constant<int, BN>{});
+        float rs_hi = pass(std::integral_constant<int, kLoKeys / 16>{},
+                           std::integral_constant<int, BN / 16>{}, -m_run);
+        float alpha = 1.f;
+        if (__any_sync(0xffffffffu, !(rs_lo + rs_hi < 256.f))) {
+          const bool wt = mbar_wait(bar(B_PL + x), j & 1, kBudgetNs, abort, gabort);
+          ok = __all_sync(0xffffffffu, wt);
+          if (!ok) break;
+          tc_fence_after();
+          const float mxs = row_max(std::integral_constant<int, kLoKeys>{}) * sc;
+          const bool move = mxs > m_run + kRescaleThreshold;
+          if (move) {
+            alpha = ex2_approx(m_run - mxs);
+            m_run = mxs;
+          }
+          if (__any_sync(0xffffffffu, move)) {
+            rescale_o(alpha);
+            rs_hi = pass(std::integral_constant<int, kLoKeys / 16>{},
+                         std::integral_constant<int, BN / 16>{}, -m_run);
           }
         }
+        tmem_st_wait();
+        l_run = alpha * (l_run + rs_lo) + rs_hi;
+        tc_fence_before();
+        mbar_arrive(bar(B_PH + x));
+      } else {
+        prep(std::integral_constant<int, kLoKeys>{}, std::integral_constant<int, BN>{});
+        const float mx = row_max(std::integral_constant<int, 0>{});
+        const float mxs = mx * sc;
+        const bool move = mx > -INFINITY && (m_run == -INFINITY || mxs > m_run + kRescaleThreshold);
+        float alpha = 1.f;
+        bool rescale = false;
+        if (move) {
+          if (m_run != -INFINITY) {
+            alpha = ex2_approx(m_run - mxs);
+            rescale = true;
+          }
+          m_run = mxs;
+        }
+        const float neg_m = m_run == -INFINITY ? 0.f : -m_run;
+        float rs;
+        if constexpr (kShort) {
+          if (short_rows && j == 0)
+            rs = pass_rem(neg_m);
+          else
+            rs = pass(std::integral_constant<int, 0>{}, std::integral_constant<int, BN / 16>{}, neg_m);
+        } else {
+          rs = pass(std::integral_constant<int, 0>{}, std::integral_constant<int, BN / 16>{}, neg_m);
+        }
+        // PV_x(j-1) is complete: this step's S-full barrier was committed after it.
+        if (__any_sync(0xffffffffu, rescale)) rescale_o(alpha);
+        tmem_st_wait();
+        l_run = l_run * alpha + rs;
+        tc_fence_before();
+        mbar_arrive(bar(B_PF + x));
+        mbar_arrive(bar(B_PH + x));
       }
-      tmem_st_wait();
-      l_run = l_run * alpha + (((sum[0].x + sum[0].y) + (sum[1].x + sum[1].y)) +
-                               ((sum[2].x + sum[2].y) + (sum[3].x + sum[3].y)));
-      tc_fence_before();
-      mbar_arrive(bar(B_PF + x));
     }
     if (!ok && r == 0) record_timeout(abort);
 

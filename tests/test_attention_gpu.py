@@ -15,11 +15,12 @@ DEV = torch.device("cuda:0") if torch.cuda.is_available() else None
 
 
 def _direct_case(kv_lens, q_lens, Hq=40, H=8, L=1, vt=False, seed=0, shuffle=True,
-                 garbage=True, vscale=1.0, order=None):
+                 garbage=True, vscale=1.0, order=None, k_edit=None):
     """Sequences written straight into a paged pool (no splice); slots past
     kv_len hold NaN so any leak of them into the output shows. vscale (a power
     of two, so exact in bf16) scales V. `order` (a permutation of the pool's
-    pages) overrides `shuffle`."""
+    pages) overrides `shuffle`. `k_edit(i, k)` may replace sequence i's K rows
+    before they are written."""
     rng = np.random.default_rng(seed)
     max_pages = max(-(-k // 16) for k in kv_lens) + 1
     n_pages = sum(-(-k // 16) for k in kv_lens) + 8
@@ -34,6 +35,8 @@ def _direct_case(kv_lens, q_lens, Hq=40, H=8, L=1, vt=False, seed=0, shuffle=Tru
         h_pt[i, :npg] = order[cur:cur + npg]
         cur += npg
         k = randn_bf16((L, T, H, 128), seed * 100 + 2 * i, DEV)
+        if k_edit is not None:
+            k = k_edit(i, k)
         v = randn_bf16((L, T, H, 128), seed * 100 + 2 * i + 1, DEV)
         if vscale != 1.0:
             v = (v.float() * vscale).to(torch.bfloat16)
@@ -210,6 +213,51 @@ def test_reprefill_equals_textbook_causal():
     nexus.reprefill(cache, d_pt, 1, mp, [T], q, o, lse, 40, 0, 1)
     assert nexus.device_status() == nexus.OK
     _check(ks, vs, q, o, lse, [T], [T], 5, what="reprefill")
+
+
+# Keys planted along a direction u that every query shares (q = (q0 + u) / 2,
+# |u|^2 = 128), so that a planted key's score a (64 +- 6) stands far above the
+# others (std ~8): the running max jumps by more than 2^8 (log2 units, 62.7 in
+# raw score) in the last 48 keys of key tile 1 (key 228: the part of P computed
+# after the first 80 keys' P is released), in the first 80 keys of tile 3 (key
+# 424), and by about the threshold in tile 4 (key 612: some rows move, some do
+# not), for every row at or after the key. One key then carries nearly all of a
+# row's weight, at up to 2^8 where the max stays, so its bf16 P alone is off by
+# up to 2^-9 of |v|: V is scaled by 1/4 to keep the outputs where 1e-2 holds
+# (a wrong rescale of O or l would miss by ~|v|).
+_PLANTED = {228: 2.0, 424: 3.5, 612: 4.6}
+
+
+@pytest.mark.parametrize("vt,split,cap", [(False, 1, None), (True, 1, None), (False, 3, None),
+                                          (True, 3, None), (False, 1, 50.0), (True, 3, 50.0)])
+def test_running_max_moves_inside_a_tile(vt, split, cap):
+    T = 640
+    g = torch.Generator().manual_seed(7)
+    u = torch.randn(128, generator=g)
+    u = u / u.norm() * 128 ** 0.5
+
+    def plant(i, k):
+        k = k.clone()
+        for key, a in _PLANTED.items():
+            k[:, key] = (a * u).to(k.dtype).to(k.device)
+        return k
+
+    cache, d_pt, mp, ks, vs, q = _direct_case([T], [T], vt=vt, seed=41 + split, k_edit=plant,
+                                              vscale=0.25)
+    q = (0.5 * q.float() + 0.5 * u.to(DEV)).to(torch.bfloat16)
+    if cap is None:
+        o, lse = _run(cache, d_pt, mp, [T], [T], q, 40, 1, split_kv=split)
+    else:
+        o = torch.full_like(q, float("nan"))
+        lse = torch.full(q.shape[:3], float("nan"), dtype=torch.float32, device=DEV)
+        nbytes, _ = nexus.attention_workspace_size([T], [T], 40, 8, 1, split)
+        ws = torch.empty(max(nbytes, 16), dtype=torch.uint8, device=DEV)
+        nexus.suffix_attention_softcap(cache, d_pt, 1, mp, [T], [T], q, o, lse, 40, 0, 1,
+                                       split_kv=split, workspace=ws, workspace_bytes=nbytes,
+                                       softcap=cap)
+        assert nexus.device_status() == nexus.OK
+    _check(ks, vs, q, o, lse, [T], [T], 5, what=f"planted maxima vt {vt} split {split} cap {cap}",
+           softcap=cap)
 
 
 def test_attention_repeat_runs_bit_stable():
