@@ -578,9 +578,10 @@ attention_kernel(const __grid_constant__ AttnLaunch p, const __grid_constant__ A
       return __all_sync(0xffffffffu, wt);
     };
     // Two issuing warps, one per query tile, in strict alternation: each waits
-    // for its own tile's P (and the K / V stages) and for the other's hand-off
-    // while the other's batch is queued, so the tensor pipe sees the single
-    // ordered stream PV_A S_A PV_B S_B ... with the waits taken off its path.
+    // for the first part of its own tile's P (and the K / V stages) and for the
+    // other's hand-off while the other's batch is queued, so the tensor pipe
+    // sees the single ordered stream PV_A S_A PV_B S_B ... with the waits taken
+    // off its path.
     // (One warp issuing both tiles spent ~1200 cycles per batch on its commits,
     // barrier polls and fence while the short product queue ran dry.) The
     // hand-off orders only the issue: every product still waits for its own
@@ -830,9 +831,9 @@ attention_kernel(const __grid_constant__ AttnLaunch p, const __grid_constant__ A
       // the issuer queues their P V products while the rest is computed. If the
       // rest moves the max (its own max is then the row's), the softmax waits
       // for those products, scales O (which then holds them) like any moved max
-      // does, and redoes the rest of P with the new max; a row whose first part
-      // already moves it (and every row's first tile) takes the max over the
-      // whole row first.
+      // does, and redoes the rest of P with the new max; a warp with a row whose
+      // first part already moves it (and every row's first tile) takes the max
+      // over the whole row first.
       prep(std::integral_constant<int, 0>{}, std::integral_constant<int, kLoKeys>{});
       const bool have_max = __all_sync(0xffffffffu, m_run != -INFINITY);
       bool fast = false;
