@@ -584,8 +584,9 @@ attention_kernel(const __grid_constant__ AttnLaunch p, const __grid_constant__ A
     // off its path.
     // (One warp issuing both tiles spent ~1200 cycles per batch on its commits,
     // barrier polls and fence while the short product queue ran dry.) The
-    // hand-off orders only the issue: every product still waits for its own
-    // data through the barriers above.
+    // hand-off orders the issue and keeps the two tiles within one batch of each
+    // other, which the K / V release barriers (one commit per tile a phase) rely
+    // on; every product still waits for its own data through the barriers above.
     const int x = warp == kMmaWarp ? 0 : 1;
     bool ok = true;
     if (n_tiles > 0 && x < n_q) {
