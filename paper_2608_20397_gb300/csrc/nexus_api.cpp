@@ -780,7 +780,8 @@ nexus_status nexus_suffix_qkv(const nexus_kv_cache* cache, const int32_t* d_page
   p->short_tiles = short_tiles ? 1 : 0;
   // A short re-decode streams the weight through few stages per CTA when each
   // tile's hidden dimension is split over a pair of CTAs (one tile per pair).
-  // Each CTA of a pair needs at least one stage of three 64-feature boxes.
+  // Each CTA of a pair needs at least one stage (two 64-feature boxes); more
+  // than three boxes in all leave each at least one.
   p->pair_split = short_tiles && 2 * n_tiles <= num_sms() && (hidden + 63) / 64 > 3 ? 1 : 0;
   double inv[kHeadDim / 2];
   fill_inv_freq_over_pi(cache, inv);

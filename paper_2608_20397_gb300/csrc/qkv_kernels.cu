@@ -73,12 +73,14 @@ struct QkvShape {
   static_assert(kSubBytes % 1024 == 0 && kABytes % 1024 == 0, "128-byte swizzle atoms");
 };
 using LongTiles = QkvShape<256, 128, 4, 1>;   // 128 tokens x two heads, 4 stages of 48 KiB
-// Up to 64 tokens x one head: 3 stages of three consecutive 64-feature boxes
-// (72 KiB), so each weight row is read 384 contiguous bytes at a time and a
-// third stage is in flight while the products consume one (two stages of four
-// boxes: 8 % slower; one box per stage, 128 bytes per row and stage: 23 %
+// Up to 64 tokens x one head: 4 stages of two consecutive 64-feature boxes
+// (48 KiB), so each weight row is read 256 contiguous bytes at a time and
+// several stages are in flight while the products consume one. A hidden size of
+// 5120 is 40 such stages, which a CTA pair splits 20 / 20 (three-box stages
+// left 14 / 13 with the last one partly past the end: 1.3 % slower; two stages of
+// four boxes: 8 % slower; one box per stage, 128 bytes per row and stage: 23 %
 // slower even with 9 stages).
-using ShortTiles = QkvShape<128, 64, 3, 3>;
+using ShortTiles = QkvShape<128, 64, 4, 2>;
 
 __device__ __forceinline__ void record_timeout(volatile int* abort) {
   *abort = 1;
