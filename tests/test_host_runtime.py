@@ -316,6 +316,20 @@ def test_workspace_size_and_split_choice():
     assert nexus.attention_workspace_size([10], [11], 40, 8, 1, 1) == (0, 0)
 
 
+def test_split_choice_matches_the_measured_optima():
+    """On 152 SMs (a GB300, and the count taken without a device) the planner
+    picks the split counts that timing sweeps on the GB300 found fastest, one
+    layer each: the c5 suffix (64 queries over 34816 keys) 10 for two-tile pairs
+    (9 for one-tile pairs, which the size query does not show), c2 (1138
+    queries over 8648 keys) 3, c3 at 25 / 50 % (548 / 1096 over 9216) 3, and
+    c3 at 100 % (2192 queries, rows that see few keys) no split."""
+    assert nexus.attention_workspace_size([34816], [64], 40, 8, 1, 0)[1] == 10
+    assert nexus.attention_workspace_size([8648], [1138], 40, 8, 1, 0)[1] == 3
+    assert nexus.attention_workspace_size([9216], [548], 40, 8, 1, 0)[1] == 3
+    assert nexus.attention_workspace_size([9216], [1096], 40, 8, 1, 0)[1] == 3
+    assert nexus.attention_workspace_size([9216], [2192], 40, 8, 1, 0)[1] == 1
+
+
 def test_zero_work_calls_succeed_before_any_launch():
     """Calls with nothing to compute return OK after validation and before any
     launch or memory access (the FAKE pointers are never dereferenced)."""
